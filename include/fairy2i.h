@@ -1,0 +1,140 @@
+/*
+ * fairy2i.h -- C ABI of the GB300 (sm_103a) Fairy2i widely-linear {+-1, +-i} layer library.
+ *
+ * The library computes the quantized widely-linear layer of Fairy2i (arXiv 2512.02901):
+ *   (1) fairy2i_convert    real map R (2n x 2m)  ->  complex pair U, W     (Sec. 3.1, Eq. UW-from-R)
+ *   (2) fairy2i_quantize   U, W -> T stages of 2-bit codes in {+-1, +-i} + per-tensor scales
+ *                          (Sec. 3.2 Eq. ifairy-proj / ifairy-scale, Sec. 3.3 residual stages,
+ *                           Sec. 3.4 2-bit storage)
+ *   (3) fairy2i_wl_matmul  y = sum_t (U^(t) x + W^(t) conj(x)), real layout in and out
+ *                          (Eq. widely-linear, Eq. res-sum, Algorithm 1)
+ *
+ * Conventions shared by every call
+ *  - Every pointer is a DEVICE pointer owned by the caller; the library keeps no pointer after
+ *    a call returns and allocates no device memory.
+ *  - `stream` is a cudaStream_t passed as void* (NULL = the legacy default stream). Calls only
+ *    enqueue work on it and never synchronize, except fairy2i_get_status.
+ *  - Argument errors are detected on the host before anything is enqueued and returned
+ *    synchronously; nothing is written in that case. A failed kernel launch returns
+ *    FAIRY2I_ERR_CUDA. Conditions found on the device (a non-finite weight, a bounded wait
+ *    that ran out) are latched in a per-device status word read by fairy2i_get_status.
+ *  - Real vectors pair their components by halves (Sec. 3.1): x~ = [Re x ; Im x]. A real
+ *    dimension that is odd is padded with one zero channel at its end (Sec. 3.1, Remarks) and
+ *    the padded output channel is discarded.
+ *  - Complex matrices are interleaved (re, im) float32 pairs (the layout of complex64).
+ */
+#ifndef FAIRY2I_H
+#define FAIRY2I_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  FAIRY2I_OK = 0,
+  FAIRY2I_ERR_INVALID_ARG = 1, /* null pointer, negative size, T out of range, bad path */
+  FAIRY2I_ERR_SHAPE = 2,       /* leading dimension smaller than the row, size mismatch */
+  FAIRY2I_ERR_ALIGNMENT = 3,   /* pointer or leading dimension breaks a stated alignment */
+  FAIRY2I_ERR_DTYPE = 4,       /* unknown activation dtype */
+  FAIRY2I_ERR_WORKSPACE = 5,   /* workspace missing or smaller than the size query */
+  FAIRY2I_ERR_NONFINITE = 6,   /* device: a weight given to fairy2i_quantize was inf or NaN */
+  FAIRY2I_ERR_TIMEOUT = 7,     /* device: a bounded wait inside a kernel ran out */
+  FAIRY2I_ERR_CUDA = 8         /* a CUDA runtime call or kernel launch failed */
+} fairy2i_status;
+
+typedef enum { FAIRY2I_F32 = 0, FAIRY2I_BF16 = 1 } fairy2i_dtype;
+
+/* Largest number of residual stages T accepted by every call. */
+#define FAIRY2I_MAX_STAGES 8
+
+/* Human-readable name of a status code (static string). */
+const char* fairy2i_status_string(fairy2i_status s);
+
+/* ------------------------------------------------------------------------------------------
+ * (1) Widely-linear conversion, Sec. 3.1 Eq. UW-from-R (proof of Theorem 1: R = R_lin(U) +
+ *     R_conj(W)).
+ *   R    float32 [rows][ldR], row-major (an nn.Linear weight: out_features x in_features).
+ *   n = ceil(rows/2), m = ceil(cols/2); R is read as a 2n x 2m matrix whose missing last row
+ *   and/or column are zero, split into n x m blocks R11 R12 / R21 R22.
+ *   U, W complex64 [n][ldc] (ldc counted in complex elements, ldc >= m):
+ *     Re U = (R11+R22)/2, Im U = (R21-R12)/2, Re W = (R11-R22)/2, Im W = (R12+R21)/2,
+ *   each computed as one float32 add/sub followed by one float32 multiply by 0.5 (IEEE
+ *   round-to-nearest-even, no contraction). Columns m..ldc-1 of U, W are not written.
+ *   Requirements: rows, cols >= 1; ldR >= cols; ldc >= m; R, U, W 4-byte aligned (U, W 8).
+ * ------------------------------------------------------------------------------------------ */
+fairy2i_status fairy2i_convert(const float* R, int64_t rows, int64_t cols, int64_t ldR,
+                               float* U, float* W, int64_t ldc, void* stream);
+
+/* ------------------------------------------------------------------------------------------
+ * (2) PhaseQuant + recursive residual quantization + 2-bit packing (Sec. 3.2-3.4).
+ *   For M in {U, W} independently: R^(0) = M; for t = 0..T-1
+ *     code c = argmax_{s in {+-1,+-i}} Re(r conj(s)) per element (Eq. ifairy-proj), ties
+ *       broken as k = floor(2 Arg(r)/pi + 1/2) breaks them, r = 0 -> +1; codeword i^c;
+ *     s_re = mean |Re r| over codes {+-1}, s_im = mean |Im r| over codes {+-i}, per tensor
+ *       (Eq. ifairy-scale); an empty set gives 0. Sums are float64 over the row-major element
+ *       order in a fixed tree (groups of 256 reduced by v[i] += v[i+h], h = 128..1, the group
+ *       sums reduced the same way until one value is left); s = float(S / N);
+ *     R^(t+1) = R^(t) - (s_re b_re + i s_im b_im) in float32, one rounding per element
+ *       (Sec. 3.3, dequantization and residual update).
+ *   U, W     complex64 [n][ldc], read only.
+ *   codes    uint32 [T][2][n][fairy2i_codes_words_per_row(m)], index 1: 0 = U, 1 = W.
+ *            Code k of a row sits in word k/16 at lane i = k%16 as two bits:
+ *              bit i    = 1 iff the codeword has Re+Im < 0  (c in {-1, -i})
+ *              bit 16+i = 1 iff the codeword has Re-Im < 0  (c in {+i, -1})
+ *            so +1 = (0,0), +i = (0,1), -1 = (1,1), -i = (1,0). Padding lanes and words are 0.
+ *            T bits per real parameter of R (Sec. 3.4) plus the row padding to 64 codes.
+ *   scales   float32 [T][2][2]: (s_re, s_im) per (stage, matrix).
+ *   workspace >= fairy2i_quantize_workspace_bytes(n, m, T) bytes of device memory, 256-byte
+ *            aligned; its contents on entry do not matter and are clobbered.
+ *   Requirements: n, m >= 1, n*m < 2^40, 1 <= T <= FAIRY2I_MAX_STAGES, ldc >= m, codes 16-byte
+ *   aligned, U, W 8-byte aligned.
+ *   A non-finite input element latches FAIRY2I_ERR_NONFINITE (the codes are then unspecified).
+ * ------------------------------------------------------------------------------------------ */
+int64_t fairy2i_codes_words_per_row(int64_t m);
+size_t fairy2i_quantize_workspace_bytes(int64_t n, int64_t m, int T);
+fairy2i_status fairy2i_quantize(const float* U, const float* W, int64_t n, int64_t m,
+                                int64_t ldc, int T, uint32_t* codes, float* scales,
+                                void* workspace, size_t workspace_bytes, void* stream);
+
+/* ------------------------------------------------------------------------------------------
+ * (3) Quantized widely-linear matmul (Eq. widely-linear with Eq. res-sum; Algorithm 1 with
+ *     the scales placed as in Eq. ifairy-dequant and the W conj(x) term included):
+ *       y_b = sum_t sum_{M in {U,W}} sum_k w^(t,M)_{jk} z_k,  z = x_b (U) or conj(x_b) (W),
+ *       w^ = s_re b_re + i s_im b_im.
+ *   x     [B][ldx] of dtype xdt (float32 or bf16): token b has in_features real entries,
+ *         Re x = x[0:m], Im x = x[m:in_features] (+ a zero if in_features is odd),
+ *         m = ceil(in_features/2).
+ *   codes, scales  as written by fairy2i_quantize for (n, m, T), n = ceil(out_features/2).
+ *   y     float32 [B][ldy], overwritten: y[0:n] = Re y, y[n:out_features] = Im y.
+ *   The result equals the float64 value of the sum up to float32 accumulation (the library
+ *   picks a memory-bound decode kernel or a tensor-core kernel by B; both accumulate in fp32).
+ *   Requirements: B >= 0 (B = 0 is a no-op), in_features, out_features >= 1, 1 <= T <= 8,
+ *   ldx >= in_features, ldy >= out_features, codes and x 16-byte aligned, y 4-byte aligned.
+ * ------------------------------------------------------------------------------------------ */
+fairy2i_status fairy2i_wl_matmul(const void* x, fairy2i_dtype xdt, int64_t B,
+                                 int64_t in_features, int64_t ldx, const uint32_t* codes,
+                                 const float* scales, int64_t out_features, int T, float* y,
+                                 int64_t ldy, void* stream);
+
+/* Same as fairy2i_wl_matmul with the kernel chosen by `path`: 0 = automatic (by B),
+ * 1 = the decode (GEMV / skinny-GEMM) kernel, 2 = the tensor-core (tcgen05) kernel.
+ * Results agree within the float32-accumulation tolerance whichever path runs. */
+fairy2i_status fairy2i_wl_matmul_path(const void* x, fairy2i_dtype xdt, int64_t B,
+                                      int64_t in_features, int64_t ldx, const uint32_t* codes,
+                                      const float* scales, int64_t out_features, int T,
+                                      float* y, int64_t ldy, int path, void* stream);
+
+/* ------------------------------------------------------------------------------------------
+ * Synchronizes `stream`, then returns and clears the device-side status of the current
+ * device: FAIRY2I_ERR_NONFINITE, FAIRY2I_ERR_TIMEOUT, FAIRY2I_ERR_CUDA (an asynchronous CUDA
+ * error) or FAIRY2I_OK.
+ * ------------------------------------------------------------------------------------------ */
+fairy2i_status fairy2i_get_status(void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* FAIRY2I_H */

@@ -1,0 +1,162 @@
+"""ctypes binding of libfairy2i.so: argument marshalling only. Every step of the path runs in
+the library's CUDA kernels; torch provides device memory and streams. There is no CPU
+fallback: a missing library raises."""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libfairy2i.so")
+
+F32, BF16 = 0, 1
+PATH_AUTO, PATH_DECODE, PATH_TENSOR = 0, 1, 2
+MAX_STAGES = 8
+STATUS = {0: "ok", 1: "invalid argument", 2: "shape", 3: "alignment", 4: "dtype", 5: "workspace",
+          6: "non-finite weight", 7: "device wait timeout", 8: "CUDA error"}
+
+_lib = None
+
+_c = ctypes
+_i64, _vp, _int, _sz = _c.c_int64, _c.c_void_p, _c.c_int, _c.c_size_t
+SIGNATURES = {
+    "fairy2i_status_string": ([_int], _c.c_char_p),
+    "fairy2i_convert": ([_vp, _i64, _i64, _i64, _vp, _vp, _i64, _vp], _int),
+    "fairy2i_codes_words_per_row": ([_i64], _i64),
+    "fairy2i_quantize_workspace_bytes": ([_i64, _i64, _int], _sz),
+    "fairy2i_quantize": ([_vp, _vp, _i64, _i64, _i64, _int, _vp, _vp, _vp, _sz, _vp], _int),
+    "fairy2i_wl_matmul": ([_vp, _int, _i64, _i64, _i64, _vp, _vp, _i64, _int, _vp, _i64, _vp],
+                          _int),
+    "fairy2i_wl_matmul_path": ([_vp, _int, _i64, _i64, _i64, _vp, _vp, _i64, _int, _vp, _i64,
+                                _int, _vp], _int),
+    "fairy2i_get_status": ([_vp], _int),
+}
+
+
+class Fairy2iError(RuntimeError):
+    def __init__(self, call: str, code: int):
+        super().__init__(f"{call}: {STATUS.get(code, code)} ({code})")
+        self.code = code
+
+
+def load(path: str = LIB_PATH):
+    """Opens the library (once). Raises if it has not been built."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(path):
+            raise RuntimeError(f"libfairy2i.so not built ({path}); run "
+                               "paper_2512_02901_gb300.build.build() first")
+        lib = ctypes.CDLL(path)
+        for name, (args, res) in SIGNATURES.items():
+            fn = getattr(lib, name)
+            fn.argtypes, fn.restype = args, res
+        _lib = lib
+    return _lib
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _check(call: str, code: int):
+    if code != 0:
+        raise Fairy2iError(call, code)
+
+
+def _ptr(t):
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def complex_dims(rows: int, cols: int):
+    return (rows + 1) // 2, (cols + 1) // 2
+
+
+def words_per_row(m: int) -> int:
+    return int(load().fairy2i_codes_words_per_row(m))
+
+
+def convert(R: torch.Tensor, stream=None):
+    """R float32 [rows][cols] (CUDA, row stride >= cols) -> U, W complex64 [n][m]."""
+    assert R.is_cuda and R.dtype == torch.float32 and R.dim() == 2 and R.stride(1) == 1
+    rows, cols = R.shape
+    n, m = complex_dims(rows, cols)
+    U = torch.empty((n, m), dtype=torch.complex64, device=R.device)
+    W = torch.empty((n, m), dtype=torch.complex64, device=R.device)
+    _check("fairy2i_convert", load().fairy2i_convert(_ptr(R), rows, cols, R.stride(0), _ptr(U),
+                                                     _ptr(W), m, _stream(stream)))
+    return U, W
+
+
+def quantize_workspace_bytes(n: int, m: int, T: int) -> int:
+    return int(load().fairy2i_quantize_workspace_bytes(n, m, T))
+
+
+def quantize(U: torch.Tensor, W: torch.Tensor, T: int, codes=None, scales=None, workspace=None,
+             stream=None):
+    """U, W complex64 [n][m] (CUDA) -> codes int32 view of uint32 [T][2][n][wpr],
+    scales float32 [T][2][2]."""
+    assert U.is_cuda and U.dtype == torch.complex64 and U.shape == W.shape and W.dtype == U.dtype
+    assert U.stride(1) == 1 and W.stride(0) == U.stride(0) and W.stride(1) == 1
+    n, m = U.shape
+    wpr = words_per_row(m)
+    dev = U.device
+    if codes is None:
+        codes = torch.empty((T, 2, n, wpr), dtype=torch.int32, device=dev)
+    if scales is None:
+        scales = torch.empty((T, 2, 2), dtype=torch.float32, device=dev)
+    nbytes = quantize_workspace_bytes(n, m, T)
+    if workspace is None or workspace.numel() < nbytes:
+        workspace = torch.empty(max(nbytes, 1), dtype=torch.uint8, device=dev)
+    _check("fairy2i_quantize",
+           load().fairy2i_quantize(_ptr(torch.view_as_real(U)), _ptr(torch.view_as_real(W)), n, m,
+                                   U.stride(0), T, _ptr(codes), _ptr(scales), _ptr(workspace),
+                                   workspace.numel(), _stream(stream)))
+    return codes, scales
+
+
+def wl_matmul(x: torch.Tensor, codes: torch.Tensor, scales: torch.Tensor, out_features: int,
+              y=None, path: int = PATH_AUTO, stream=None):
+    """x [B][in_features] float32/bf16 -> y float32 [B][out_features] = [Re y | Im y].
+    A CPU x is copied to the device (pinned staging) and y copied back: the end-to-end form."""
+    if not x.is_cuda:
+        dev = codes.device
+        xd = x.pin_memory().to(dev, non_blocking=True) if not x.is_pinned() else x.to(dev, non_blocking=True)
+        yd = wl_matmul(xd, codes, scales, out_features, path=path, stream=stream)
+        out = torch.empty(yd.shape, dtype=yd.dtype, pin_memory=True) if y is None else y
+        out.copy_(yd, non_blocking=True)
+        torch.cuda.current_stream(dev).synchronize() if stream is None else stream.synchronize()
+        return out
+    assert x.dim() == 2 and x.stride(1) == 1 and x.dtype in (torch.float32, torch.bfloat16)
+    B, in_features = x.shape
+    T = codes.shape[0]
+    if y is None:
+        y = torch.empty((B, out_features), dtype=torch.float32, device=x.device)
+    xdt = F32 if x.dtype == torch.float32 else BF16
+    _check("fairy2i_wl_matmul",
+           load().fairy2i_wl_matmul_path(_ptr(x), xdt, B, in_features, x.stride(0), _ptr(codes),
+                                         _ptr(scales), out_features, T, _ptr(y), y.stride(0),
+                                         path, _stream(stream)))
+    return y
+
+
+def get_status(stream=None) -> int:
+    """Synchronizes the stream and returns (and clears) the device-side status code."""
+    return int(load().fairy2i_get_status(_stream(stream)))
+
+
+class Fairy2iLinear:
+    """A real linear layer (weight [out][in], fp32) converted and quantized once; calls run the
+    quantized widely-linear matmul."""
+
+    def __init__(self, weight: torch.Tensor, T: int = 2):
+        self.out_features, self.in_features = weight.shape
+        self.T = T
+        U, W = convert(weight)
+        self.codes, self.scales = quantize(U, W, T)
+
+    def __call__(self, x: torch.Tensor, path: int = PATH_AUTO) -> torch.Tensor:
+        return wl_matmul(x, self.codes, self.scales, self.out_features, path=path)

@@ -1,0 +1,147 @@
+// C ABI of the library: argument validation, the per-device status word, dispatch.
+#include <cuda_runtime.h>
+
+#include <mutex>
+
+#include "common.cuh"
+
+namespace fairy2i {
+
+fairy2i_status launch_convert(const float* R, int64_t rows, int64_t cols, int64_t ldR, int64_t n,
+                              int64_t m, float* U, float* W, int64_t ldc, cudaStream_t stream);
+size_t quantize_workspace_bytes(int64_t n, int64_t m);
+fairy2i_status launch_quantize(const float* U, const float* W, int64_t n, int64_t m, int64_t ldc,
+                               int T, uint32_t* codes, float* scales, void* workspace,
+                               cudaStream_t stream);
+fairy2i_status launch_wl_simple(const void* x, fairy2i_dtype xdt, int64_t B, int64_t in_features,
+                                int64_t ldx, const uint32_t* codes, const float* scales,
+                                int64_t n, int64_t m, int64_t out_features, int64_t wpr, int T,
+                                float* y, int64_t ldy, cudaStream_t stream);
+fairy2i_status launch_wl_decode(const void* x, fairy2i_dtype xdt, int64_t B, int64_t in_features,
+                                int64_t ldx, const uint32_t* codes, const float* scales,
+                                int64_t n, int64_t m, int64_t out_features, int64_t wpr, int T,
+                                float* y, int64_t ldy, cudaStream_t stream, bool* handled);
+
+// Status word: one __device__ word per device that has loaded the module; its address is
+// looked up once per device with that device current.
+__device__ unsigned int g_status_word;
+static unsigned int* g_status_ptr[64];
+static std::mutex g_status_mu;
+
+unsigned int* device_status_word() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  std::lock_guard<std::mutex> lock(g_status_mu);
+  if (!g_status_ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_status_word) != cudaSuccess) return nullptr;
+    g_status_ptr[dev] = static_cast<unsigned int*>(p);
+  }
+  return g_status_ptr[dev];
+}
+
+static bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+}  // namespace fairy2i
+
+using namespace fairy2i;
+
+extern "C" {
+
+const char* fairy2i_status_string(fairy2i_status s) {
+  switch (s) {
+    case FAIRY2I_OK: return "ok";
+    case FAIRY2I_ERR_INVALID_ARG: return "invalid argument";
+    case FAIRY2I_ERR_SHAPE: return "shape or leading dimension error";
+    case FAIRY2I_ERR_ALIGNMENT: return "misaligned pointer or leading dimension";
+    case FAIRY2I_ERR_DTYPE: return "unknown dtype";
+    case FAIRY2I_ERR_WORKSPACE: return "workspace missing or too small";
+    case FAIRY2I_ERR_NONFINITE: return "non-finite weight";
+    case FAIRY2I_ERR_TIMEOUT: return "bounded wait ran out on the device";
+    case FAIRY2I_ERR_CUDA: return "CUDA error";
+  }
+  return "unknown status";
+}
+
+fairy2i_status fairy2i_convert(const float* R, int64_t rows, int64_t cols, int64_t ldR, float* U,
+                               float* W, int64_t ldc, void* stream) {
+  if (!R || !U || !W || rows < 1 || cols < 1) return FAIRY2I_ERR_INVALID_ARG;
+  const int64_t n = (rows + 1) / 2, m = (cols + 1) / 2;
+  if (ldR < cols || ldc < m) return FAIRY2I_ERR_SHAPE;
+  if (!aligned(R, 4) || !aligned(U, 8) || !aligned(W, 8)) return FAIRY2I_ERR_ALIGNMENT;
+  return launch_convert(R, rows, cols, ldR, n, m, U, W, ldc, static_cast<cudaStream_t>(stream));
+}
+
+int64_t fairy2i_codes_words_per_row(int64_t m) { return m < 1 ? 0 : ((m + 63) / 64) * 4; }
+
+size_t fairy2i_quantize_workspace_bytes(int64_t n, int64_t m, int T) {
+  if (n < 1 || m < 1 || T < 1 || T > FAIRY2I_MAX_STAGES) return 0;
+  return quantize_workspace_bytes(n, m);
+}
+
+fairy2i_status fairy2i_quantize(const float* U, const float* W, int64_t n, int64_t m, int64_t ldc,
+                                int T, uint32_t* codes, float* scales, void* workspace,
+                                size_t workspace_bytes, void* stream) {
+  if (!U || !W || !codes || !scales || n < 1 || m < 1 || T < 1 || T > FAIRY2I_MAX_STAGES)
+    return FAIRY2I_ERR_INVALID_ARG;
+  if (n > (int64_t(1) << 40) / m) return FAIRY2I_ERR_SHAPE;
+  if (ldc < m) return FAIRY2I_ERR_SHAPE;
+  if (!aligned(U, 8) || !aligned(W, 8) || !aligned(codes, 16) || !aligned(scales, 4))
+    return FAIRY2I_ERR_ALIGNMENT;
+  if (!workspace || workspace_bytes < quantize_workspace_bytes(n, m)) return FAIRY2I_ERR_WORKSPACE;
+  if (!aligned(workspace, 256)) return FAIRY2I_ERR_ALIGNMENT;
+  return launch_quantize(U, W, n, m, ldc, T, codes, scales, workspace,
+                         static_cast<cudaStream_t>(stream));
+}
+
+fairy2i_status fairy2i_wl_matmul_path(const void* x, fairy2i_dtype xdt, int64_t B,
+                                      int64_t in_features, int64_t ldx, const uint32_t* codes,
+                                      const float* scales, int64_t out_features, int T, float* y,
+                                      int64_t ldy, int path, void* stream) {
+  if (B < 0 || in_features < 1 || out_features < 1 || T < 1 || T > FAIRY2I_MAX_STAGES ||
+      path < 0 || path > 2)
+    return FAIRY2I_ERR_INVALID_ARG;
+  if (xdt != FAIRY2I_F32 && xdt != FAIRY2I_BF16) return FAIRY2I_ERR_DTYPE;
+  if (B == 0) return FAIRY2I_OK;
+  if (!x || !codes || !scales || !y) return FAIRY2I_ERR_INVALID_ARG;
+  if (ldx < in_features || ldy < out_features) return FAIRY2I_ERR_SHAPE;
+  if (!aligned(x, 16) || !aligned(codes, 16) || !aligned(y, 4) || !aligned(scales, 4))
+    return FAIRY2I_ERR_ALIGNMENT;
+  const int64_t n = (out_features + 1) / 2, m = (in_features + 1) / 2;
+  const int64_t wpr = fairy2i_codes_words_per_row(m);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (path == 2) return FAIRY2I_ERR_INVALID_ARG;  // tensor-core path not built in this library
+  bool handled = false;
+  fairy2i_status st = launch_wl_decode(x, xdt, B, in_features, ldx, codes, scales, n, m,
+                                       out_features, wpr, T, y, ldy, s, &handled);
+  if (handled || st != FAIRY2I_OK) return st;
+  return launch_wl_simple(x, xdt, B, in_features, ldx, codes, scales, n, m, out_features, wpr, T,
+                          y, ldy, s);
+}
+
+fairy2i_status fairy2i_wl_matmul(const void* x, fairy2i_dtype xdt, int64_t B, int64_t in_features,
+                                 int64_t ldx, const uint32_t* codes, const float* scales,
+                                 int64_t out_features, int T, float* y, int64_t ldy,
+                                 void* stream) {
+  return fairy2i_wl_matmul_path(x, xdt, B, in_features, ldx, codes, scales, out_features, T, y,
+                                ldy, 0, stream);
+}
+
+fairy2i_status fairy2i_get_status(void* stream) {
+  if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess)
+    return FAIRY2I_ERR_CUDA;
+  unsigned int* p = device_status_word();
+  if (!p) return FAIRY2I_ERR_CUDA;
+  unsigned int v = 0;
+  if (cudaMemcpy(&v, p, sizeof(v), cudaMemcpyDeviceToHost) != cudaSuccess) return FAIRY2I_ERR_CUDA;
+  if (v) {
+    const unsigned int zero = 0;
+    if (cudaMemcpy(p, &zero, sizeof(zero), cudaMemcpyHostToDevice) != cudaSuccess)
+      return FAIRY2I_ERR_CUDA;
+  }
+  if (v & kStatusTimeout) return FAIRY2I_ERR_TIMEOUT;
+  if (v & kStatusNonfinite) return FAIRY2I_ERR_NONFINITE;
+  return FAIRY2I_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,52 @@
+// Shared device helpers of the Fairy2i sm_103a kernels.
+#pragma once
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "fairy2i.h"
+
+namespace fairy2i {
+
+// Bits latched in the per-device status word.
+enum : unsigned int { kStatusNonfinite = 1u, kStatusTimeout = 2u };
+
+// Code values: codeword i^c, c = 0:+1, 1:+i, 2:-1, 3:-i.
+// PhaseQuant projection (Eq. ifairy-proj): the larger of |Re r|, |Im r| with its sign wins;
+// ties |Re r| = |Im r| != 0 take the codeword counter-clockwise of the diagonal (the choice of
+// k = floor(2 Arg(r)/pi + 1/2)); r = 0 gives +1. Comparisons treat -0 as +0.
+__device__ __forceinline__ unsigned project_code(float a, float b) {
+  const float aa = fabsf(a), ab = fabsf(b);
+  if (aa > ab) return a > 0.f ? 0u : 2u;
+  if (ab > aa) return b > 0.f ? 1u : 3u;
+  if (aa == 0.f) return 0u;
+  if (b > 0.f) return a > 0.f ? 1u : 2u;
+  return a < 0.f ? 3u : 0u;
+}
+
+// Residual update of Sec. 3.3: r -= s_re b_re + i s_im b_im, one IEEE add per element.
+__device__ __forceinline__ void residual_update(float& a, float& b, unsigned c, float s_re,
+                                                float s_im) {
+  if (c == 0u) a = __fsub_rn(a, s_re);
+  else if (c == 2u) a = __fadd_rn(a, s_re);
+  else if (c == 1u) b = __fsub_rn(b, s_im);
+  else b = __fadd_rn(b, s_im);
+}
+
+// Packed bit pair of a code: (Re+Im < 0, Re-Im < 0) of the codeword.
+__device__ __forceinline__ unsigned neg_sum_bit(unsigned c) { return c >> 1; }            // 2,3
+__device__ __forceinline__ unsigned neg_diff_bit(unsigned c) { return (c ^ (c >> 1)) & 1u; }  // 1,2
+
+__device__ __forceinline__ void latch_status(unsigned int* status, unsigned int bit) {
+  if (status) atomicOr(status, bit);
+}
+
+}  // namespace fairy2i
+
+// Launch helpers shared by the host-side launchers.
+namespace fairy2i {
+inline fairy2i_status launch_status() {
+  return cudaGetLastError() == cudaSuccess ? FAIRY2I_OK : FAIRY2I_ERR_CUDA;
+}
+// Per-device status word (defined in api.cu).
+unsigned int* device_status_word();
+}  // namespace fairy2i

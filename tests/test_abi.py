@@ -1,0 +1,93 @@
+"""The C-ABI library builds, loads and exports every symbol its header declares; host-side
+argument validation returns its errors synchronously (no GPU needed: nothing is enqueued)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import __graft_entry__ as entry
+from paper_2512_02901_gb300 import binding as F
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "fairy2i.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    entry.build()
+    return F.load()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(fairy2i_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_header_declares_the_three_calls():
+    names = declared_functions()
+    for n in ("fairy2i_convert", "fairy2i_quantize", "fairy2i_wl_matmul", "fairy2i_get_status"):
+        assert n in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+        assert name in F.SIGNATURES, f"binding lacks a signature for {name}"
+
+
+def test_status_strings(lib):
+    for code in range(9):
+        assert lib.fairy2i_status_string(code)
+
+
+def test_size_queries(lib):
+    assert lib.fairy2i_codes_words_per_row(1) == 4
+    assert lib.fairy2i_codes_words_per_row(64) == 4
+    assert lib.fairy2i_codes_words_per_row(65) == 8
+    assert lib.fairy2i_codes_words_per_row(5504) == 344
+    assert lib.fairy2i_codes_words_per_row(0) == 0
+    assert lib.fairy2i_quantize_workspace_bytes(2048, 2048, 2) > 0
+    assert lib.fairy2i_quantize_workspace_bytes(2048, 2048, 0) == 0
+    assert lib.fairy2i_quantize_workspace_bytes(2048, 2048, 9) == 0
+
+
+P = ctypes.c_void_p
+GOOD = P(1 << 20)            # a 16-byte aligned non-null stand-in; never dereferenced
+ODD = P((1 << 20) + 4)
+
+
+def test_convert_validation(lib):
+    assert lib.fairy2i_convert(None, 4, 4, 4, GOOD, GOOD, 2, None) == 1
+    assert lib.fairy2i_convert(GOOD, 0, 4, 4, GOOD, GOOD, 2, None) == 1
+    assert lib.fairy2i_convert(GOOD, 4, 4, 3, GOOD, GOOD, 2, None) == 2       # ldR < cols
+    assert lib.fairy2i_convert(GOOD, 4, 5, 5, GOOD, GOOD, 2, None) == 2       # ldc < m = 3
+    assert lib.fairy2i_convert(GOOD, 4, 4, 4, ODD, GOOD, 2, None) == 3        # U not 8-aligned
+
+
+def test_quantize_validation(lib):
+    ws = lib.fairy2i_quantize_workspace_bytes(8, 8, 2)
+    args = dict(U=GOOD, W=GOOD, n=8, m=8, ldc=8, T=2, codes=GOOD, scales=GOOD, ws=GOOD, wsb=ws)
+
+    def call(**kw):
+        a = dict(args, **kw)
+        return lib.fairy2i_quantize(a["U"], a["W"], a["n"], a["m"], a["ldc"], a["T"], a["codes"],
+                                    a["scales"], a["ws"], a["wsb"], None)
+    assert call(T=0) == 1 and call(T=9) == 1 and call(U=None) == 1 and call(n=0) == 1
+    assert call(ldc=7) == 2
+    assert call(codes=ODD) == 3
+    assert call(wsb=ws - 1) == 5 and call(ws=None) == 5
+    assert call(ws=P((1 << 20) + 16)) == 3                                     # not 256-aligned
+
+
+def test_wl_matmul_validation(lib):
+    def call(x=GOOD, xdt=1, B=1, inf=16, ldx=16, codes=GOOD, scales=GOOD, outf=16, T=2, y=GOOD,
+             ldy=16, path=0):
+        return lib.fairy2i_wl_matmul_path(x, xdt, B, inf, ldx, codes, scales, outf, T, y, ldy,
+                                          path, None)
+    assert call(B=0) == 0                      # empty batch: nothing to do
+    assert call(B=-1) == 1 and call(T=0) == 1 and call(path=3) == 1 and call(x=None) == 1
+    assert call(xdt=7) == 4
+    assert call(ldx=15) == 2 and call(ldy=15) == 2
+    assert call(x=ODD) == 3 and call(codes=ODD) == 3

@@ -1,0 +1,245 @@
+"""GPU parity: the CUDA library (through its C ABI) against the CPU oracle on the same seeded
+inputs. Conversion, codes and scales must match bit for bit; matmul outputs must satisfy
+relative Frobenius error <= 1e-5 and |err| <= 1e-4 * ||x~||_1 * sum_t s_t per element, where
+sum_t s_t = sum over stages of max(s_re, s_im) of U plus that of W."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2512_02901_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+REL_FRO = 1e-5
+ELEM = 1e-4
+
+
+@pytest.fixture(scope="module")
+def F():
+    import __graft_entry__ as entry
+    entry.build()
+    from paper_2512_02901_gb300 import binding
+    binding.load()
+    return binding
+
+
+DEV = "cuda:0"
+
+
+def _np_codes(codes_t):
+    return codes_t.cpu().numpy().view(np.uint32)
+
+
+def assert_wl_close(yg, yo, x, scales, rows=None):
+    yg = np.asarray(yg, dtype=np.float64)
+    err = yg - yo
+    denom = np.linalg.norm(yo)
+    rel = np.linalg.norm(err) / denom if denom > 0 else np.linalg.norm(err)
+    assert rel <= REL_FRO, f"relative Frobenius error {rel:.3e}"
+    bound = ELEM * O.tolerance_bound(np.asarray(x, np.float64), scales)[:, None]
+    worst = np.max(np.abs(err) - bound)
+    assert worst <= 0, f"element error exceeds bound by {worst:.3e}"
+
+
+def upload_codes(packed):
+    return torch.from_numpy(np.ascontiguousarray(packed).view(np.int32)).to(DEV)
+
+
+# ------------------------------------------------------------------------------ convert
+@pytest.mark.parametrize("rows,cols", [(256, 256), (7, 9), (1, 1), (3, 130), (4096, 4096),
+                                       (11008, 4096), (4096, 11008)])
+def test_convert_bit_exact(F, rows, cols):
+    R = synth.random_matrix(rows, cols, seed=rows * 7 + cols, scale=0.02)
+    U, W = F.convert(R.to(DEV))
+    Uo, Wo = O.convert(R.numpy())
+    assert np.array_equal(U.cpu().numpy().view(np.uint64), Uo.view(np.uint64))
+    assert np.array_equal(W.cpu().numpy().view(np.uint64), Wo.view(np.uint64))
+
+
+def test_convert_strided_input(F):
+    base = synth.random_matrix(10, 40, seed=5)
+    R = base[:, 3:20]                                    # ldR = 40 > cols = 17
+    U, W = F.convert(base.to(DEV)[:, 3:20])
+    Uo, Wo = O.convert(R.contiguous().numpy())
+    assert np.array_equal(U.cpu().numpy(), Uo) and np.array_equal(W.cpu().numpy(), Wo)
+
+
+# ------------------------------------------------------------------------------ quantize
+def _quantize_both(F, U_np, W_np, T):
+    U = torch.from_numpy(U_np).to(DEV)
+    W = torch.from_numpy(W_np).to(DEV)
+    codes, scales = F.quantize(U, W, T)
+    assert F.get_status() == 0
+    co, so = O.quantize(U_np, W_np, T)
+    return codes, scales, co, so
+
+
+def _assert_quant_equal(codes, scales, co, so):
+    got = _np_codes(codes)
+    want = O.pack_codes(co)
+    assert got.shape == want.shape
+    mism = np.argwhere(got != want)
+    assert mism.size == 0, f"{len(mism)} packed words differ, first at {mism[:3].tolist()}"
+    gs = scales.cpu().numpy()
+    assert np.array_equal(gs.view(np.uint32), so.view(np.uint32)), (gs, so)
+
+
+@pytest.mark.parametrize("n,m,T", [(128, 128, 2), (37, 53, 3), (1, 1, 1), (5, 65, 2), (300, 17, 4),
+                                   (64, 200, 8)])
+def test_quantize_bit_exact_small(F, n, m, T):
+    g = np.random.default_rng(n * 1000 + m)
+    U = (0.02 * g.standard_normal((n, m)) + 0.02j * g.standard_normal((n, m))).astype(np.complex64)
+    W = (0.02 * g.standard_normal((n, m)) + 0.02j * g.standard_normal((n, m))).astype(np.complex64)
+    _assert_quant_equal(*_quantize_both(F, U, W, T))
+
+
+def test_quantize_tiny_layer_bit_exact(F):
+    A, _ = synth.tiny_layer()
+    U, W = F.convert(A.to(DEV))
+    codes, scales = F.quantize(U, W, 2)
+    Uo, Wo = O.convert(A.numpy())
+    co, so = O.quantize(Uo, Wo, 2)
+    _assert_quant_equal(codes, scales, co, so)
+
+
+def test_quantize_ties_zero_and_degenerate(F):
+    """Exact ties, signed zeros, an all-zero matrix (empty +-i set -> s_im = 0)."""
+    vals = np.array([1, -1, 0.5, -0.5, 0.0, -0.0, 2.0], dtype=np.float32)
+    g = np.random.default_rng(7)
+    re = g.choice(vals, size=(19, 33)).astype(np.float32)
+    im = np.where(g.random((19, 33)) < 0.5, re, -re).astype(np.float32)
+    U = (re + 1j * im).astype(np.complex64)
+    W = np.zeros((19, 33), dtype=np.complex64)
+    codes, scales, co, so = _quantize_both(F, U, W, 3)
+    _assert_quant_equal(codes, scales, co, so)
+    assert so[0, 1, 1] == 0.0
+
+
+def test_quantize_strided_rows(F):
+    g = np.random.default_rng(11)
+    big = (g.standard_normal((20, 80)) + 1j * g.standard_normal((20, 80))).astype(np.complex64)
+    Ud = torch.from_numpy(big).to(DEV)[:, :70]
+    Wd = torch.from_numpy(big[:, ::-1].copy()).to(DEV)[:, :70]
+    codes, scales = F.quantize(Ud, Wd, 2)
+    co, so = O.quantize(big[:, :70], big[:, ::-1][:, :70], 2)
+    _assert_quant_equal(codes, scales, co, so)
+
+
+def test_quantize_nonfinite_latches_status(F):
+    U = torch.zeros((4, 16), dtype=torch.complex64, device=DEV)
+    U[1, 3] = complex(float("nan"), 0.0)
+    W = torch.ones((4, 16), dtype=torch.complex64, device=DEV)
+    F.quantize(U, W, 1)
+    assert F.get_status() == 6
+    assert F.get_status() == 0          # read clears
+
+
+@pytest.mark.parametrize("rows,cols,T,seed", [
+    (4096, 4096, 2, synth.weight_seed("attn")),             # attention projection, decode
+    (11008, 4096, 2, synth.weight_seed("mlp", 0)),          # up / gate
+    (4096, 11008, 2, synth.weight_seed("mlp", 2)),          # down
+    (11008, 4096, 3, synth.weight_seed("prefill", 0)),
+    (4096, 11008, 1, synth.weight_seed("prefill", 1)),
+])
+def test_quantize_bit_exact_full_size(F, rows, cols, T, seed):
+    R = synth.student_t_weight(rows, cols, seed)
+    U, W = F.convert(R.to(DEV))
+    codes, scales = F.quantize(U, W, T)
+    assert F.get_status() == 0
+    Uo, Wo = O.convert(R.numpy())
+    co, so = O.quantize(Uo, Wo, T)
+    _assert_quant_equal(codes, scales, co, so)
+
+
+# ------------------------------------------------------------------------------ wl_matmul
+def _random_quantized(n, m, T, seed):
+    g = np.random.default_rng(seed)
+    codes = g.integers(0, 4, (T, 2, n, m)).astype(np.uint8)
+    scales = (0.01 + 0.02 * g.random((T, 2, 2))).astype(np.float32)
+    return codes, scales
+
+
+def _run_wl(F, x_t, codes, scales, out_features, path=0):
+    y = F.wl_matmul(x_t.to(DEV), upload_codes(O.pack_codes(codes)),
+                    torch.from_numpy(scales).to(DEV), out_features, path=path)
+    assert F.get_status() == 0
+    return y.cpu().numpy()
+
+
+def test_wl_tiny_layer_fp32(F):
+    A, x = synth.tiny_layer()
+    Uo, Wo = O.convert(A.numpy())
+    co, so = O.quantize(Uo, Wo, 2)
+    yg = _run_wl(F, x, co, so, 256)
+    yo = O.wl_matmul(x.numpy(), co, so, 256)
+    assert_wl_close(yg, yo, x.numpy(), so)
+
+
+@pytest.mark.parametrize("out_f,in_f,T,B,dtype", [
+    (8, 8, 1, 1, torch.float32), (37, 53, 2, 3, torch.float32), (37, 53, 3, 5, torch.bfloat16),
+    (130, 258, 2, 17, torch.bfloat16), (1, 1, 1, 2, torch.float32), (2, 129, 8, 4, torch.bfloat16),
+    (255, 1001, 2, 1, torch.bfloat16), (1024, 96, 2, 64, torch.bfloat16),
+])
+def test_wl_matmul_shapes(F, out_f, in_f, T, B, dtype):
+    n, m = O.complex_dims(out_f, in_f)
+    codes, scales = _random_quantized(n, m, T, seed=out_f * 31 + in_f)
+    x = synth.random_matrix(B, in_f, seed=B + in_f).to(dtype)
+    yg = _run_wl(F, x, codes, scales, out_f)
+    xo = x.float().numpy()
+    yo = O.wl_matmul(xo, codes, scales, out_f)
+    assert_wl_close(yg, yo, xo, scales)
+
+
+def test_wl_matmul_strided_x_and_y(F):
+    n, m, T, B = 40, 24, 2, 6
+    codes, scales = _random_quantized(n, m, T, seed=3)
+    xbig = synth.random_matrix(B, 2 * m + 16, seed=9).to(torch.bfloat16)
+    x = xbig.to(DEV)[:, : 2 * m]
+    y = torch.full((B, 2 * n + 8), 7.0, device=DEV)
+    F.wl_matmul(x, upload_codes(O.pack_codes(codes)), torch.from_numpy(scales).to(DEV), 2 * n,
+                y=y[:, : 2 * n])
+    yg = y.cpu().numpy()
+    assert np.all(yg[:, 2 * n:] == 7.0)                      # beyond out_features untouched
+    xo = xbig[:, : 2 * m].float().numpy()
+    assert_wl_close(yg[:, : 2 * n], O.wl_matmul(xo, codes, scales, 2 * n), xo, scales)
+
+
+def _layer(rows, cols, T, seed):
+    R = synth.student_t_weight(rows, cols, seed)
+    Uo, Wo = O.convert(R.numpy())
+    co, so = O.quantize(Uo, Wo, T)
+    return co, so
+
+
+@pytest.mark.parametrize("rows,cols,B,seed", [
+    (4096, 4096, 1, synth.weight_seed("attn")),
+    (11008, 4096, 1, synth.weight_seed("mlp", 0)),
+    (11008, 4096, 4, synth.weight_seed("mlp", 1)),
+    (4096, 11008, 16, synth.weight_seed("mlp", 2)),
+])
+def test_wl_matmul_full_size_decode(F, rows, cols, B, seed):
+    co, so = _layer(rows, cols, 2, seed)
+    x = synth.outlier_activations(B, cols, synth.activation_seed(seed, B))
+    yg = _run_wl(F, x, co, so, rows)
+    xo = x.float().numpy()
+    yo = O.wl_matmul(xo, co, so, rows)
+    assert_wl_close(yg, yo, xo, so)
+
+
+@pytest.mark.parametrize("rows,cols,T", [(11008, 4096, 1), (4096, 11008, 3)])
+def test_wl_matmul_prefill_sampled(F, rows, cols, T):
+    """2048 tokens; the oracle computes a sample of 96 output rows for every token."""
+    seed = synth.weight_seed("prefill", 0 if rows > cols else 1)
+    co, so = _layer(rows, cols, T, seed)
+    B = 2048
+    x = synth.outlier_activations(B, cols, synth.activation_seed(seed, B))
+    yg = _run_wl(F, x, co, so, rows)
+    n, m = co.shape[2], co.shape[3]
+    g = np.random.default_rng(0)
+    rws = np.sort(g.choice(n, 96, replace=False))
+    xo = x.float().numpy()
+    yc = O.wl_matmul_rows(O.split_input(xo, m), co, so, rws)
+    yo = np.concatenate([yc.real, yc.imag], axis=1)
+    ys = np.concatenate([yg[:, rws], yg[:, n + rws]], axis=1)
+    assert_wl_close(ys, yo, xo, so)
