@@ -100,6 +100,31 @@ fairy2i_status fairy2i_quantize(const float* U, const float* W, int64_t n, int64
                                 void* workspace, size_t workspace_bytes, void* stream);
 
 /* ------------------------------------------------------------------------------------------
+ * fairy2i_quantize without a workspace argument. The paper has no counterpart: this is a
+ * convenience for callers that cannot allocate device memory at the point of the call, such as
+ * a plugin inside a host framework that owns every byte of device memory through its own pool
+ * (a raw cudaMalloc there may fail, and a cudaFree synchronizes the whole device), or a
+ * latency-bound caller that may not put an allocation on its call path.
+ *
+ * Same arguments and results as fairy2i_quantize, minus the workspace. The scratch lives in a
+ * fixed device array of FAIRY2I_NOALLOC_SCRATCH_BYTES (4 MiB) inside the library, which every
+ * GPU that loads the library holds until the process exits. The call allocates nothing and
+ * calls no allocating routine.
+ *  - Sizes: fairy2i_quantize_workspace_bytes(n, m, T) must not exceed the array, i.e.
+ *    n*m <= 16,646,656 complex weights per matrix (a 4096 -> 11008 layer, 5504 x 2048, fits);
+ *    larger sizes return FAIRY2I_ERR_WORKSPACE and enqueue nothing.
+ *  - The first call on a device looks up the array's device address (cudaGetSymbolAddress,
+ *    with that device current); make that first call before any stream capture on the device.
+ *  - All calls share the one array, on every stream: calls whose kernels overlap on the GPU
+ *    (different streams without ordering between them) race and give wrong results. Calls
+ *    ordered on one stream are safe; each call writes every scratch entry before reading it.
+ * ------------------------------------------------------------------------------------------ */
+#define FAIRY2I_NOALLOC_SCRATCH_BYTES (4u << 20)
+fairy2i_status fairy2i_quantize_noalloc(const float* U, const float* W, int64_t n, int64_t m,
+                                        int64_t ldc, int T, uint32_t* codes, float* scales,
+                                        void* stream);
+
+/* ------------------------------------------------------------------------------------------
  * (3) Quantized widely-linear matmul (Eq. widely-linear with Eq. res-sum; Algorithm 1 with
  *     the scales placed as in Eq. ifairy-dequant and the W conj(x) term included):
  *       y_b = sum_t sum_{M in {U,W}} sum_k w^(t,M)_{jk} z_k,  z = x_b (U) or conj(x_b) (W),

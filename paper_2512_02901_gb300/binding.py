@@ -32,6 +32,7 @@ SIGNATURES = {
     "fairy2i_wl_matmul_path": ([_vp, _int, _i64, _i64, _i64, _vp, _vp, _i64, _int, _vp, _i64,
                                 _int, _vp], _int),
     "fairy2i_get_status": ([_vp], _int),
+    "fairy2i_quantize_noalloc": ([_vp, _vp, _i64, _i64, _i64, _int, _vp, _vp, _vp], _int),
 }
 
 
