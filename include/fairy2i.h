@@ -80,12 +80,17 @@ fairy2i_status fairy2i_convert(const float* R, int64_t rows, int64_t cols, int64
  *     R^(t+1) = R^(t) - (s_re b_re + i s_im b_im) in float32, one rounding per element
  *       (Sec. 3.3, dequantization and residual update).
  *   U, W     complex64 [n][ldc], read only.
- *   codes    uint32 [T][2][n][fairy2i_codes_words_per_row(m)], index 1: 0 = U, 1 = W.
- *            Code k of a row sits in word k/16 at lane i = k%16 as two bits:
- *              bit i    = 1 iff the codeword has Re+Im < 0  (c in {-1, -i})
- *              bit 16+i = 1 iff the codeword has Re-Im < 0  (c in {+i, -1})
- *            so +1 = (0,0), +i = (0,1), -1 = (1,1), -i = (1,0). Padding lanes and words are 0.
- *            T bits per real parameter of R (Sec. 3.4) plus the row padding to 64 codes.
+ *   codes    fairy2i_codes_words(n, m, T) uint32 words. Each row of codes is padded with zero
+ *            codes to wpr = fairy2i_codes_words_per_row(m) words (16 codes per word, rows
+ *            padded to 128 codes) and the rows to 16 R (R = ceil(n/16)) with zero rows; the
+ *            buffer is uint32 [T][2][R][wpr/8][16 rows][8 words] (index 1: 0 = U, 1 = W), i.e.
+ *            every block of 16 rows x 128 codes is 512 contiguous bytes.
+ *            Code k of a row sits in word k/16 at lane i = k%16 as two bits, at
+ *            b(i) = 8 (i%2) + i/2 (even codes fill byte 0, odd codes byte 1, in order):
+ *              bit b(i)    = 1 iff the codeword has Re+Im < 0  (c in {-1, -i})
+ *              bit 16+b(i) = 1 iff the codeword has Re-Im < 0  (c in {+i, -1})
+ *            so +1 = (0,0), +i = (0,1), -1 = (1,1), -i = (1,0). Padding is code +1 (0 bits).
+ *            T bits per real parameter of R (Sec. 3.4) plus the padding.
  *   scales   float32 [T][2][2]: (s_re, s_im) per (stage, matrix).
  *   workspace >= fairy2i_quantize_workspace_bytes(n, m, T) bytes of device memory, 256-byte
  *            aligned; its contents on entry do not matter and are clobbered.
@@ -94,6 +99,7 @@ fairy2i_status fairy2i_convert(const float* R, int64_t rows, int64_t cols, int64
  *   A non-finite input element latches FAIRY2I_ERR_NONFINITE (the codes are then unspecified).
  * ------------------------------------------------------------------------------------------ */
 int64_t fairy2i_codes_words_per_row(int64_t m);
+int64_t fairy2i_codes_words(int64_t n, int64_t m, int T);
 size_t fairy2i_quantize_workspace_bytes(int64_t n, int64_t m, int T);
 fairy2i_status fairy2i_quantize(const float* U, const float* W, int64_t n, int64_t m,
                                 int64_t ldc, int T, uint32_t* codes, float* scales,

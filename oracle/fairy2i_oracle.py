@@ -35,8 +35,8 @@ import numpy as np
 
 __all__ = [
     "complex_dims", "convert", "realify_lin", "realify_conj", "project", "fixed_tree_sum",
-    "axis_scales", "dequant", "residual_quantize", "quantize", "words_per_row", "pack_codes",
-    "unpack_codes", "split_input", "wl_matmul", "wl_matmul_rows", "dense_realified",
+    "axis_scales", "dequant", "residual_quantize", "quantize", "words_per_row", "row_tiles",
+    "pack_codes", "unpack_codes", "split_input", "wl_matmul", "wl_matmul_rows", "dense_realified",
     "tolerance_bound",
 ]
 
@@ -222,40 +222,62 @@ def quantize(U, W, T: int, mode: str = "contract"):
 # Sec. 3.4 -- 2-bit storage
 # --------------------------------------------------------------------------------------------
 def words_per_row(m: int) -> int:
-    """32-bit words per packed code row: 16 codes per word, rows padded to 64 codes."""
-    return -(-m // 64) * 4
+    """32-bit words per packed code row: 16 codes per word, rows padded to 128 codes."""
+    return -(-m // 128) * 8
+
+
+def row_tiles(n: int) -> int:
+    """Packed rows come in tiles of 16 (the last one zero-padded)."""
+    return -(-n // 16)
+
+
+def _bit_of_lane(i):
+    """Bit of the (Re+Im<0) flag of code i (0..15) inside its word: even codes fill byte 0,
+    odd codes byte 1, in order; the (Re-Im<0) flag sits 16 bits higher."""
+    return 8 * (i & 1) + (i >> 1)
 
 
 def pack_codes(codes):
-    """2 bits per complex weight (Sec. 3.4, storage). Layout, uint32 [T][2][n][words_per_row(m)]:
-    code k of a row lives in word k // 16 at lane i = k % 16, as two bits
-        bit i      = 1 iff c in {2, 3}   (the codeword has Re + Im < 0)
-        bit 16 + i = 1 iff c in {1, 2}   (the codeword has Re - Im < 0)
-    Padding lanes and words are zero (which is code 0)."""
+    """2 bits per complex weight (Sec. 3.4, storage).
+
+    Word format: the 16 codes i = 0..15 of a word (code k of a row: word k // 16, i = k % 16)
+    each own two bits,
+        bit b(i)      = 1 iff c in {2, 3}   (the codeword has Re + Im < 0)
+        bit 16 + b(i) = 1 iff c in {1, 2}   (the codeword has Re - Im < 0)
+    with b(i) = 8 (i % 2) + i // 2: byte 0 holds the first flag of the even codes, byte 1 of
+    the odd codes, bytes 2 and 3 the second flag likewise.
+    Buffer order: codes [T][2][n][m] are padded to [T][2][16 R][8 C words] (R = row_tiles(n),
+    C = words_per_row(m) / 8; padding codes are 0) and stored as
+    uint32 [T][2][R][C][16 rows][8 words]: a 16-row x 128-code block is 512 contiguous bytes.
+    Returns a flat uint32 array."""
     codes = np.asarray(codes, dtype=np.uint32)
-    lead, m = codes.shape[:-1], codes.shape[-1]
+    T, two, n, m = codes.shape
     wpr = words_per_row(m)
-    full = np.zeros(lead + (wpr * 16,), dtype=np.uint32)
-    full[..., :m] = codes
-    full = full.reshape(lead + (wpr, 16))
-    neg_sum = ((full == 2) | (full == 3)).astype(np.uint32)
-    neg_diff = ((full == 1) | (full == 2)).astype(np.uint32)
-    lane = np.arange(16, dtype=np.uint32)
-    words = (neg_sum << lane).sum(axis=-1, dtype=np.uint64) + \
-        (neg_diff << (lane + 16)).sum(axis=-1, dtype=np.uint64)
-    return words.astype(np.uint32)
+    R = row_tiles(n)
+    full = np.zeros((T, two, R * 16, wpr * 16), dtype=np.uint32)
+    full[:, :, :n, :m] = codes
+    full = full.reshape(T, two, R * 16, wpr, 16)
+    neg_sum = ((full == 2) | (full == 3)).astype(np.uint64)
+    neg_diff = ((full == 1) | (full == 2)).astype(np.uint64)
+    bit = np.array([_bit_of_lane(i) for i in range(16)], dtype=np.uint64)
+    words = ((neg_sum << bit) + (neg_diff << (bit + 16))).sum(axis=-1).astype(np.uint32)
+    words = words.reshape(T, two, R, 16, wpr // 8, 8).transpose(0, 1, 2, 4, 3, 5)
+    return np.ascontiguousarray(words).reshape(-1)
 
 
-def unpack_codes(words, m: int):
-    """Inverse of ``pack_codes``: uint8 codes [..., m]."""
-    words = np.asarray(words, dtype=np.uint32)
-    lane = np.arange(16, dtype=np.uint32)
-    neg_sum = (words[..., None] >> lane) & 1
-    neg_diff = (words[..., None] >> (lane + 16)) & 1
+def unpack_codes(words, T: int, n: int, m: int):
+    """Inverse of ``pack_codes``: uint8 codes [T][2][n][m]."""
+    wpr = words_per_row(m)
+    R = row_tiles(n)
+    w = np.asarray(words, dtype=np.uint32).reshape(T, 2, R, wpr // 8, 16, 8)
+    w = w.transpose(0, 1, 2, 4, 3, 5).reshape(T, 2, R * 16, wpr)
+    bit = np.array([_bit_of_lane(i) for i in range(16)], dtype=np.uint32)
+    neg_sum = (w[..., None] >> bit) & 1
+    neg_diff = (w[..., None] >> (bit + 16)) & 1
     # (neg_sum, neg_diff): (0,0) -> 0, (0,1) -> 1, (1,1) -> 2, (1,0) -> 3
     c = np.where(neg_sum == 0, neg_diff, 3 - neg_diff)
-    c = c.reshape(words.shape[:-1] + (words.shape[-1] * 16,))
-    return c[..., :m].astype(np.uint8)
+    c = c.reshape(T, 2, R * 16, wpr * 16)
+    return c[:, :, :n, :m].astype(np.uint8)
 
 
 # --------------------------------------------------------------------------------------------

@@ -25,6 +25,7 @@ SIGNATURES = {
     "fairy2i_status_string": ([_int], _c.c_char_p),
     "fairy2i_convert": ([_vp, _i64, _i64, _i64, _vp, _vp, _i64, _vp], _int),
     "fairy2i_codes_words_per_row": ([_i64], _i64),
+    "fairy2i_codes_words": ([_i64, _i64, _int], _i64),
     "fairy2i_quantize_workspace_bytes": ([_i64, _i64, _int], _sz),
     "fairy2i_quantize": ([_vp, _vp, _i64, _i64, _i64, _int, _vp, _vp, _vp, _sz, _vp], _int),
     "fairy2i_wl_matmul": ([_vp, _int, _i64, _i64, _i64, _vp, _vp, _i64, _int, _vp, _i64, _vp],
@@ -98,15 +99,15 @@ def quantize_workspace_bytes(n: int, m: int, T: int) -> int:
 
 def quantize(U: torch.Tensor, W: torch.Tensor, T: int, codes=None, scales=None, workspace=None,
              stream=None):
-    """U, W complex64 [n][m] (CUDA) -> codes int32 view of uint32 [T][2][n][wpr],
-    scales float32 [T][2][2]."""
+    """U, W complex64 [n][m] (CUDA) -> codes: int32 view of the packed uint32 words,
+    shape [T][2][ceil(n/16)][wpr/8][16][8]; scales float32 [T][2][2]."""
     assert U.is_cuda and U.dtype == torch.complex64 and U.shape == W.shape and W.dtype == U.dtype
     assert U.stride(1) == 1 and W.stride(0) == U.stride(0) and W.stride(1) == 1
     n, m = U.shape
     wpr = words_per_row(m)
     dev = U.device
     if codes is None:
-        codes = torch.empty((T, 2, n, wpr), dtype=torch.int32, device=dev)
+        codes = torch.empty((T, 2, (n + 15) // 16, wpr // 8, 16, 8), dtype=torch.int32, device=dev)
     if scales is None:
         scales = torch.empty((T, 2, 2), dtype=torch.float32, device=dev)
     nbytes = quantize_workspace_bytes(n, m, T)
@@ -120,20 +121,21 @@ def quantize(U: torch.Tensor, W: torch.Tensor, T: int, codes=None, scales=None, 
 
 
 def wl_matmul(x: torch.Tensor, codes: torch.Tensor, scales: torch.Tensor, out_features: int,
-              y=None, path: int = PATH_AUTO, stream=None):
+              y=None, path: int = PATH_AUTO, stream=None, T: int | None = None):
     """x [B][in_features] float32/bf16 -> y float32 [B][out_features] = [Re y | Im y].
     A CPU x is copied to the device (pinned staging) and y copied back: the end-to-end form."""
     if not x.is_cuda:
         dev = codes.device
         xd = x.pin_memory().to(dev, non_blocking=True) if not x.is_pinned() else x.to(dev, non_blocking=True)
-        yd = wl_matmul(xd, codes, scales, out_features, path=path, stream=stream)
+        yd = wl_matmul(xd, codes, scales, out_features, path=path, stream=stream, T=T)
         out = torch.empty(yd.shape, dtype=yd.dtype, pin_memory=True) if y is None else y
         out.copy_(yd, non_blocking=True)
         torch.cuda.current_stream(dev).synchronize() if stream is None else stream.synchronize()
         return out
     assert x.dim() == 2 and x.stride(1) == 1 and x.dtype in (torch.float32, torch.bfloat16)
     B, in_features = x.shape
-    T = codes.shape[0]
+    if T is None:
+        T = scales.shape[0]
     if y is None:
         y = torch.empty((B, out_features), dtype=torch.float32, device=x.device)
     xdt = F32 if x.dtype == torch.float32 else BF16

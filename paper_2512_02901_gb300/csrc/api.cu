@@ -72,7 +72,12 @@ fairy2i_status fairy2i_convert(const float* R, int64_t rows, int64_t cols, int64
   return launch_convert(R, rows, cols, ldR, n, m, U, W, ldc, static_cast<cudaStream_t>(stream));
 }
 
-int64_t fairy2i_codes_words_per_row(int64_t m) { return m < 1 ? 0 : ((m + 63) / 64) * 4; }
+int64_t fairy2i_codes_words_per_row(int64_t m) { return m < 1 ? 0 : ((m + 127) / 128) * 8; }
+
+int64_t fairy2i_codes_words(int64_t n, int64_t m, int T) {
+  if (n < 1 || m < 1 || T < 1 || T > FAIRY2I_MAX_STAGES) return 0;
+  return (int64_t)T * 2 * ((n + 15) / 16) * 16 * fairy2i_codes_words_per_row(m);
+}
 
 size_t fairy2i_quantize_workspace_bytes(int64_t n, int64_t m, int T) {
   if (n < 1 || m < 1 || T < 1 || T > FAIRY2I_MAX_STAGES) return 0;

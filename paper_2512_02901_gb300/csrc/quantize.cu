@@ -132,20 +132,29 @@ __global__ void __launch_bounds__(512) quant_reduce_kernel(const double* partial
   }
 }
 
-// One warp per (matrix, row); 32 consecutive codes per iteration -> ballots -> two words per
-// stage: word0 = (neg_sum lanes 0-15) | (neg_diff lanes 0-15) << 16, word1 likewise for 16-31.
-__global__ void __launch_bounds__(256) quant_pack_kernel(QuantArgs q, int64_t wpr,
+// One warp per (matrix, row) of the padded row range (16 rows per tile); 32 consecutive codes
+// per iteration -> ballots -> two words per stage: word0 = (neg_sum lanes 0-15) |
+// (neg_diff lanes 0-15) << 16, word1 likewise for lanes 16-31, with the lanes permuted so
+// that each ballot bit lands at its code's bit. Words are stored in
+// [T][2][row tile][chunk of 8 words][16 rows][8 words] order; rows >= n are written as 0.
+__global__ void __launch_bounds__(256) quant_pack_kernel(QuantArgs q, int64_t wpr, int64_t tiles,
                                                          uint32_t* __restrict__ codes) {
   const int lane = threadIdx.x & 31;
+  const int64_t rows = tiles * 16;
   const int64_t row = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
-  if (row >= 2 * q.n) return;
-  const int mat = (int)(row / q.n);
-  const int64_t j = row - (int64_t)mat * q.n;
-  const float2* __restrict__ Mrow = (mat ? q.M[1] : q.M[0]) + j * q.ldc;
+  if (row >= 2 * rows) return;
+  const int mat = (int)(row / rows);
+  const int64_t j = row - (int64_t)mat * rows;
+  const bool live_row = j < q.n;
+  const float2* __restrict__ Mrow = (mat ? q.M[1] : q.M[0]) + (live_row ? j : 0) * q.ldc;
+  const int64_t chunks = wpr / 8;
+  // Lane l handles code i = 2 (l % 8) + (l / 8) % 2 of word w + l / 16, so that the ballot bit
+  // of lane l is bit 8 (i % 2) + i / 2 of the word (even codes in byte 0, odd codes in byte 1).
+  const int code_of_lane = (lane >> 4) * 16 + 2 * (lane & 7) + ((lane >> 3) & 1);
   for (int64_t w = 0; w < wpr; w += 2) {
-    const int64_t k = w * 16 + lane;
+    const int64_t k = w * 16 + code_of_lane;
     float a = 0.f, b = 0.f;
-    const bool live = k < q.m;
+    const bool live = live_row && k < q.m;
     if (live) { const float2 r = Mrow[k]; a = r.x; b = r.y; }
     for (int t = 0; t < q.T; ++t) {
       const unsigned c = project_code(a, b);
@@ -154,7 +163,10 @@ __global__ void __launch_bounds__(256) quant_pack_kernel(QuantArgs q, int64_t wp
       if (lane < 2) {
         const uint32_t word = lane == 0 ? ((ns & 0xffffu) | (nd << 16))
                                         : ((ns >> 16) | (nd & 0xffff0000u));
-        codes[(((int64_t)t * 2 + mat) * q.n + j) * wpr + w + lane] = word;
+        const int64_t ww = w + lane;
+        const int64_t idx = ((((int64_t)t * 2 + mat) * tiles + j / 16) * chunks + ww / 8) * 128 +
+                            (j % 16) * 8 + ww % 8;
+        codes[idx] = word;
       }
       residual_update(a, b, c, __ldg(q.scales + (t * 2 + mat) * 2 + 0),
                       __ldg(q.scales + (t * 2 + mat) * 2 + 1));
@@ -190,7 +202,8 @@ fairy2i_status launch_quantize(const float* U, const float* W, int64_t n, int64_
     if (cudaGetLastError() != cudaSuccess) return FAIRY2I_ERR_CUDA;
   }
   const int64_t wpr = fairy2i_codes_words_per_row(m);
-  quant_pack_kernel<<<(unsigned)ceil_div(2 * n, 8), 256, 0, stream>>>(q, wpr, codes);
+  const int64_t tiles = ceil_div(n, 16);
+  quant_pack_kernel<<<(unsigned)ceil_div(2 * tiles * 16, 8), 256, 0, stream>>>(q, wpr, tiles, codes);
   return launch_status();
 }
 

@@ -46,17 +46,21 @@ __global__ void __launch_bounds__(256) wl_simple_kernel(WlArgs a) {
   for (int b = 0; b < NB; ++b) yr[b] = yi[b] = 0.f;
 
   for (int tm = 0; tm < 2 * a.T; ++tm) {
-    const uint32_t* __restrict__ row = a.codes + ((int64_t)tm * a.n + j) * a.wpr;
+    // [T][2][row tile][chunk][16 rows][8 words] packing
+    const int64_t tiles = (a.n + 15) / 16, chunks = a.wpr / 8;
+    const uint32_t* __restrict__ row =
+        a.codes + (((int64_t)tm * tiles + j / 16) * chunks) * 128 + (j % 16) * 8;
     float pr[NB], pi[NB], qr[NB], qi[NB];
 #pragma unroll
     for (int b = 0; b < NB; ++b) pr[b] = pi[b] = qr[b] = qi[b] = 0.f;
     for (int64_t w = lane; w < a.wpr; w += 32) {
-      const uint32_t word = __ldg(row + w);
+      const uint32_t word = __ldg(row + (w / 8) * 128 + (w % 8));
       for (int i = 0; i < 16; ++i) {
         const int64_t k = w * 16 + i;
         if (k >= a.m) break;
-        const uint32_t sneg = ((word >> i) & 1u) << 31;
-        const uint32_t tneg = ((word >> (16 + i)) & 1u) << 31;
+        const int bit = 8 * (i & 1) + (i >> 1);     // even codes in byte 0, odd in byte 1
+        const uint32_t sneg = ((word >> bit) & 1u) << 31;
+        const uint32_t tneg = ((word >> (16 + bit)) & 1u) << 31;
 #pragma unroll
         for (int b = 0; b < NB; ++b) {
           const int64_t bb = b0 + b;

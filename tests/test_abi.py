@@ -43,10 +43,12 @@ def test_status_strings(lib):
 
 
 def test_size_queries(lib):
-    assert lib.fairy2i_codes_words_per_row(1) == 4
-    assert lib.fairy2i_codes_words_per_row(64) == 4
-    assert lib.fairy2i_codes_words_per_row(65) == 8
+    assert lib.fairy2i_codes_words_per_row(1) == 8
+    assert lib.fairy2i_codes_words_per_row(128) == 8
+    assert lib.fairy2i_codes_words_per_row(129) == 16
     assert lib.fairy2i_codes_words_per_row(5504) == 344
+    assert lib.fairy2i_codes_words(5504, 2048, 2) == 2 * 2 * 5504 * 128
+    assert lib.fairy2i_codes_words(17, 1, 1) == 2 * 32 * 8
     assert lib.fairy2i_codes_words_per_row(0) == 0
     assert lib.fairy2i_quantize_workspace_bytes(2048, 2048, 2) > 0
     assert lib.fairy2i_quantize_workspace_bytes(2048, 2048, 0) == 0

@@ -28,7 +28,7 @@ DEV = "cuda:0"
 
 
 def _np_codes(codes_t):
-    return codes_t.cpu().numpy().view(np.uint32)
+    return codes_t.cpu().numpy().view(np.uint32).reshape(-1)
 
 
 def assert_wl_close(yg, yo, x, scales, rows=None):
@@ -243,3 +243,31 @@ def test_wl_matmul_prefill_sampled(F, rows, cols, T):
     yo = np.concatenate([yc.real, yc.imag], axis=1)
     ys = np.concatenate([yg[:, rws], yg[:, n + rws]], axis=1)
     assert_wl_close(ys, yo, xo, so)
+
+
+@pytest.mark.parametrize("out_f,in_f,T,B", [
+    (32, 32, 1, 1), (31, 515, 2, 2), (4096, 4096, 4, 1), (100, 8192, 3, 2), (17, 2, 2, 1),
+    (4096, 11008, 2, 2), (11008, 4096, 2, 1), (48, 1024, 2, 2),
+])
+def test_wl_decode_path(F, out_f, in_f, T, B):
+    """The decode path (tensor-core GEMV for B <= 2 bf16 tokens) on ragged rows and chunks."""
+    n, m = O.complex_dims(out_f, in_f)
+    codes, scales = _random_quantized(n, m, T, seed=out_f + 7 * in_f + T)
+    x = synth.outlier_activations(B, in_f, seed=out_f + in_f)
+    yg = _run_wl(F, x, codes, scales, out_f, path=1)
+    xo = x.float().numpy()
+    assert_wl_close(yg, O.wl_matmul(xo, codes, scales, out_f), xo, scales)
+
+
+def test_wl_decode_all_codes_each_value(F):
+    """Every code value in every word position (catches a wrong position class)."""
+    n, m, T = 16, 256, 1
+    codes = np.zeros((T, 2, n, m), dtype=np.uint8)
+    for j in range(n):
+        codes[0, 0, j] = (np.arange(m) + j) % 4
+        codes[0, 1, j] = (np.arange(m) // 16 + 3 * j) % 4
+    scales = np.array([[[0.03, 0.011], [0.017, 0.029]]], dtype=np.float32)
+    x = synth.outlier_activations(1, 2 * m, seed=99)
+    yg = _run_wl(F, x, codes, scales, 2 * n, path=1)
+    xo = x.float().numpy()
+    assert_wl_close(yg, O.wl_matmul(xo, codes, scales, 2 * n), xo, scales)

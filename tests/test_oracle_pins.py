@@ -265,19 +265,27 @@ def test_single_weight_closed_form():
 
 # ---------------------------------------------------------------- Sec. 3.4, storage
 def test_packed_layout_hand_word():
-    c = np.zeros((1, 1, 1, 16), dtype=np.uint8)
-    c[..., :4] = [0, 1, 2, 3]
+    c = np.zeros((1, 2, 17, 140), dtype=np.uint8)
+    c[0, 0, 0, :4] = [0, 1, 2, 3]
+    c[0, 1, 16, 130] = 2                     # W, row 16 (second row tile), code 130
     w = O.pack_codes(c)
-    # Re+Im < 0 for codes 2, 3 (lanes 2, 3); Re-Im < 0 for codes 1, 2 (lanes 1, 2)
-    assert w.shape == (1, 1, 1, 4) and w[0, 0, 0, 0] == 0x0006000C and not np.any(w[..., 1:])
+    # 2 matrices x 2 row tiles x 2 chunks x 16 rows x 8 words
+    assert w.shape == (2 * 2 * 2 * 128,)
+    # Re+Im < 0 for codes 2, 3 -> bits 1 (even code 2) and 9 (odd code 3);
+    # Re-Im < 0 for codes 1, 2 -> bits 16+8 (odd code 1) and 16+1 (even code 2)
+    assert w[0] == 0x01020202
+    # W (block 4), row tile 1, chunk 1 (codes 128..255), row 0, word 0, lane 2
+    idx = (((1 * 2 + 1) * 2 + 1) * 16 + 0) * 8 + 0
+    assert w[idx] == (1 << 1) | (1 << 17)
+    assert np.count_nonzero(w) == 2
 
 
-@pytest.mark.parametrize("T,n,m", [(1, 4, 64), (2, 8, 128), (3, 5, 77)])
+@pytest.mark.parametrize("T,n,m", [(1, 16, 128), (2, 32, 256), (3, 5, 77), (2, 17, 129)])
 def test_storage_is_T_bits_per_real_parameter(T, n, m):
     c = rng.integers(0, 4, (T, 2, n, m)).astype(np.uint8)
     w = O.pack_codes(c)
-    assert np.array_equal(O.unpack_codes(w, m), c)
-    if m % 64 == 0:
+    assert np.array_equal(O.unpack_codes(w, T, n, m), c)
+    if m % 128 == 0 and n % 16 == 0:
         assert w.nbytes * 8 == T * (2 * n) * (2 * m)     # T bits per real parameter of R
 
 
