@@ -21,6 +21,10 @@ fairy2i_status launch_wl_decode(const void* x, fairy2i_dtype xdt, int64_t B, int
                                 int64_t ldx, const uint32_t* codes, const float* scales,
                                 int64_t n, int64_t m, int64_t out_features, int64_t wpr, int T,
                                 float* y, int64_t ldy, cudaStream_t stream, bool* handled);
+fairy2i_status launch_wl_tc(const void* x, fairy2i_dtype xdt, int64_t B, int64_t in_features,
+                            int64_t ldx, const uint32_t* codes, const float* scales, int64_t n,
+                            int64_t m, int64_t out_features, int64_t wpr, int T, float* y,
+                            int64_t ldy, cudaStream_t stream, bool* handled);
 
 // Status word: one __device__ word per device that has loaded the module; its address is
 // looked up once per device with that device current.
@@ -115,9 +119,15 @@ fairy2i_status fairy2i_wl_matmul_path(const void* x, fairy2i_dtype xdt, int64_t 
   const int64_t n = (out_features + 1) / 2, m = (in_features + 1) / 2;
   const int64_t wpr = fairy2i_codes_words_per_row(m);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if (path == 2) return FAIRY2I_ERR_INVALID_ARG;  // tensor-core path not built in this library
   bool handled = false;
-  fairy2i_status st = launch_wl_decode(x, xdt, B, in_features, ldx, codes, scales, n, m,
+  fairy2i_status st = FAIRY2I_OK;
+  if (path == 2) {   // tcgen05 decode kernel (explicit): B <= 2 bf16 tokens, T <= 4
+    st = launch_wl_tc(x, xdt, B, in_features, ldx, codes, scales, n, m, out_features, wpr, T, y,
+                      ldy, s, &handled);
+    if (handled || st != FAIRY2I_OK) return st;
+    return FAIRY2I_ERR_INVALID_ARG;   // shape or dtype outside the tcgen05 decode kernel
+  }
+  st = launch_wl_decode(x, xdt, B, in_features, ldx, codes, scales, n, m,
                                        out_features, wpr, T, y, ldy, s, &handled);
   if (handled || st != FAIRY2I_OK) return st;
   return launch_wl_simple(x, xdt, B, in_features, ldx, codes, scales, n, m, out_features, wpr, T,

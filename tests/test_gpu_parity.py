@@ -271,3 +271,65 @@ def test_wl_decode_all_codes_each_value(F):
     yg = _run_wl(F, x, codes, scales, 2 * n, path=1)
     xo = x.float().numpy()
     assert_wl_close(yg, O.wl_matmul(xo, codes, scales, 2 * n), xo, scales)
+
+
+# ------------------------------------------------------------------------------ tcgen05 decode
+@pytest.mark.parametrize("out_f,in_f,T,B", [
+    (32, 32, 1, 1), (31, 515, 2, 2), (64, 256, 3, 1), (4096, 4096, 4, 1), (100, 8192, 3, 2),
+    (17, 2, 2, 1), (4096, 11008, 2, 2), (11008, 4096, 2, 1), (48, 1024, 2, 2),
+    (4096, 4096, 2, 1), (130, 45056, 2, 1),
+])
+def test_wl_tcgen05_decode_path(F, out_f, in_f, T, B):
+    """The tcgen05 decode kernel (path 2) on ragged rows and chunks, every T it takes, clusters of
+    1..8 CTAs per row block (in_features 45056: 176 chunks, 8 CTAs of 22), odd in_features (x
+    staged by plain loads) and 16-byte-aligned rows (x staged by bulk copy)."""
+    n, m = O.complex_dims(out_f, in_f)
+    codes, scales = _random_quantized(n, m, T, seed=3 * out_f + 5 * in_f + T)
+    x = synth.outlier_activations(B, in_f, seed=out_f + in_f + 1)
+    yg = _run_wl(F, x, codes, scales, out_f, path=2)
+    xo = x.float().numpy()
+    assert_wl_close(yg, O.wl_matmul(xo, codes, scales, out_f), xo, scales)
+
+
+@pytest.mark.parametrize("T", [1, 2, 3, 4])
+def test_wl_tcgen05_all_codes_each_value(F, T):
+    """Every code value at every word position of every stage-matrix lane block."""
+    n, m = 40, 384
+    codes = np.zeros((T, 2, n, m), dtype=np.uint8)
+    for t in range(T):
+        for j in range(n):
+            codes[t, 0, j] = (np.arange(m) + j + t) % 4
+            codes[t, 1, j] = (np.arange(m) // 16 + 3 * j + t) % 4
+    g = np.random.default_rng(T)
+    scales = (0.01 + 0.02 * g.random((T, 2, 2))).astype(np.float32)
+    x = synth.outlier_activations(2, 2 * m, seed=7 + T)
+    yg = _run_wl(F, x, codes, scales, 2 * n, path=2)
+    xo = x.float().numpy()
+    assert_wl_close(yg, O.wl_matmul(xo, codes, scales, 2 * n), xo, scales)
+
+
+def test_wl_tcgen05_strided_x_and_y(F):
+    n, m, T, B = 70, 136, 2, 2
+    codes, scales = _random_quantized(n, m, T, seed=11)
+    xbig = synth.outlier_activations(B, 2 * m + 24, seed=12)
+    x = xbig.to(DEV)[:, : 2 * m]
+    y = torch.full((B, 2 * n + 8), 7.0, device=DEV)
+    F.wl_matmul(x, upload_codes(O.pack_codes(codes)), torch.from_numpy(scales).to(DEV), 2 * n,
+                y=y[:, : 2 * n], path=2)
+    assert F.get_status() == 0
+    yg = y.cpu().numpy()
+    assert np.all(yg[:, 2 * n:] == 7.0)
+    xo = xbig[:, : 2 * m].float().numpy()
+    assert_wl_close(yg[:, : 2 * n], O.wl_matmul(xo, codes, scales, 2 * n), xo, scales)
+
+
+def test_wl_tcgen05_rejects_outside_its_domain(F):
+    n, m, T = 16, 64, 2
+    codes, scales = _random_quantized(n, m, T, seed=13)
+    cd = upload_codes(O.pack_codes(codes))
+    sc = torch.from_numpy(scales).to(DEV)
+    for x in (synth.outlier_activations(3, 2 * m, seed=1).to(DEV),          # B = 3
+              torch.zeros((1, 2 * m), dtype=torch.float32, device=DEV)):    # fp32 x
+        with pytest.raises(F.Fairy2iError) as e:
+            F.wl_matmul(x, cd, sc, 2 * n, path=2)
+        assert e.value.code == 1
