@@ -151,12 +151,16 @@ fairy2i_status fairy2i_wl_matmul(const void* x, fairy2i_dtype xdt, int64_t B,
                                  int64_t ldy, void* stream);
 
 /* Same as fairy2i_wl_matmul with the kernel chosen by `path`:
- *   0 = automatic: the warp-MMA decode kernel for B <= 2 bf16 tokens and T <= 4, otherwise the
- *       general kernel;
- *   1 = the same choice as 0 (the decode kernel where it applies);
+ *   0 = automatic: B <= 2 bf16 tokens and T <= 4 -> the warp-MMA decode kernel; B > 2 -> the
+ *       tcgen05 prefill GEMM where it applies (see 3); otherwise the general CUDA-core kernel;
+ *   1 = the decode kernel where it applies, otherwise the general kernel;
  *   2 = the tcgen05 decode kernel (5th-generation tensor cores, the code matrix in tensor
  *       memory); it takes B <= 2 bf16 tokens, T <= 4 and rows of at most 176 128-code chunks
- *       (in_features <= 45056) and returns FAIRY2I_ERR_INVALID_ARG for anything else.
+ *       (in_features <= 45056) and returns FAIRY2I_ERR_INVALID_ARG for anything else;
+ *   3 = the tcgen05 prefill GEMM (codes expanded into bf16 +-1 tiles in tensor memory, x by TMA,
+ *       64 tokens per tile); it takes bf16 x with 16-byte aligned rows, ldx % 8 == 0,
+ *       m % 8 == 0 (m = ceil(in_features/2)) and T <= 4, and returns FAIRY2I_ERR_INVALID_ARG for
+ *       anything else.
  * Results agree within the float32-accumulation tolerance whichever path runs. */
 fairy2i_status fairy2i_wl_matmul_path(const void* x, fairy2i_dtype xdt, int64_t B,
                                       int64_t in_features, int64_t ldx, const uint32_t* codes,

@@ -12,7 +12,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libfairy2i.so")
 
 F32, BF16 = 0, 1
-PATH_AUTO, PATH_DECODE, PATH_TENSOR = 0, 1, 2
+PATH_AUTO, PATH_DECODE, PATH_TC_DECODE, PATH_TC_PREFILL = 0, 1, 2, 3
 MAX_STAGES = 8
 STATUS = {0: "ok", 1: "invalid argument", 2: "shape", 3: "alignment", 4: "dtype", 5: "workspace",
           6: "non-finite weight", 7: "device wait timeout", 8: "CUDA error"}

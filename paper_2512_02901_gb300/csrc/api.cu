@@ -25,6 +25,10 @@ fairy2i_status launch_wl_tc(const void* x, fairy2i_dtype xdt, int64_t B, int64_t
                             int64_t ldx, const uint32_t* codes, const float* scales, int64_t n,
                             int64_t m, int64_t out_features, int64_t wpr, int T, float* y,
                             int64_t ldy, cudaStream_t stream, bool* handled);
+fairy2i_status launch_wl_prefill(const void* x, fairy2i_dtype xdt, int64_t B, int64_t in_features,
+                                 int64_t ldx, const uint32_t* codes, const float* scales,
+                                 int64_t n, int64_t m, int64_t out_features, int64_t wpr, int T,
+                                 float* y, int64_t ldy, cudaStream_t stream, bool* handled);
 
 // Status word: one __device__ word per device that has loaded the module; its address is
 // looked up once per device with that device current.
@@ -108,7 +112,7 @@ fairy2i_status fairy2i_wl_matmul_path(const void* x, fairy2i_dtype xdt, int64_t 
                                       const float* scales, int64_t out_features, int T, float* y,
                                       int64_t ldy, int path, void* stream) {
   if (B < 0 || in_features < 1 || out_features < 1 || T < 1 || T > FAIRY2I_MAX_STAGES ||
-      path < 0 || path > 2)
+      path < 0 || path > 3)
     return FAIRY2I_ERR_INVALID_ARG;
   if (xdt != FAIRY2I_F32 && xdt != FAIRY2I_BF16) return FAIRY2I_ERR_DTYPE;
   if (B == 0) return FAIRY2I_OK;
@@ -121,6 +125,12 @@ fairy2i_status fairy2i_wl_matmul_path(const void* x, fairy2i_dtype xdt, int64_t 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   bool handled = false;
   fairy2i_status st = FAIRY2I_OK;
+  if (path == 3 || (path == 0 && B > 2)) {   // tcgen05 prefill GEMM
+    st = launch_wl_prefill(x, xdt, B, in_features, ldx, codes, scales, n, m, out_features, wpr, T,
+                           y, ldy, s, &handled);
+    if (handled || st != FAIRY2I_OK) return st;
+    if (path == 3) return FAIRY2I_ERR_INVALID_ARG;   // outside the prefill kernel's domain
+  }
   if (path == 2) {   // tcgen05 decode kernel (explicit): B <= 2 bf16 tokens, T <= 4
     st = launch_wl_tc(x, xdt, B, in_features, ldx, codes, scales, n, m, out_features, wpr, T, y,
                       ldy, s, &handled);

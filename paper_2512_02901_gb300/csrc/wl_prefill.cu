@@ -1,0 +1,496 @@
+// Prefill (many-token) kernel of the quantized widely-linear matmul on the 5th-generation tensor
+// cores: a GEMM whose weight operand is expanded from the 2-bit codes on the fly.
+//
+// Arithmetic (Eq. ifairy-dequant, Algorithm 1 with the W conj(x) term): with sigma = sign(Re b +
+// Im b), tau = sign(Re b - Im b) of the codeword b and h = (s_re + i s_im)/2, the dequantized
+// weight is h sigma + conj(h) tau, so per (stage t, matrix) and output row the layer needs the +-1
+// sums P = sum_k sigma_k x_k and Q = sum_k tau_k x_k; y += h P + conj(h) Q for U and
+// h conj(P) + conj(h) conj(Q) for W. +-1 and bf16 x are exact in a bf16 x bf16 -> f32 MMA.
+//
+// GEMM form. Tile = one row block (R rows of every stage-matrix: TMEM lane tm*R + r, R = 64, 32,
+// 16, 16 for T = 1..4) x 64 tokens. Per 16 codes (one code word per lane) two tcgen05.mma
+// kind::f16 (M = 128, N = 128, K = 16) run: A = the sigma (or tau) plane of the word as bf16 +-1 in
+// tensor memory, B = x of the 64 tokens (rows 0-63: Re x, rows 64-127: Im x) in shared memory, D =
+// the sigma accumulator (TMEM columns 0-127) or the tau accumulator (128-255): column p*64 + b is
+// the sum for part p (re/im) of token b. x arrives by TMA (128-byte swizzle, one box of 64 codes x
+// 64 tokens per part; Re and Im through two tensor maps so that each part is zero beyond its end).
+// The CTAs are persistent over the tiles, ordered token-tile-major so that CTAs running together
+// share x in L2.
+//
+// Roles (11 warps): warps 0-7, two sets of four (warp w reaches TMEM lanes 32 (w % 4) ..), decode
+// the code words into the TMEM A ring, set s taking the step pairs p = s (mod 2) (one 32-column
+// store per pair: sigma, tau of two steps of 16 codes), and run the epilogue of each tile, set s for
+// tokens 32 s .. 32 s + 31; warps 8 and 9 issue the sigma and the tau MMAs (one commit per pair
+// each); warp 10 copies the codes (bulk copies of whole 16-row tiles) and x (TMA) in.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_bf16.h>
+
+#include <mutex>
+
+#include "common.cuh"
+#include "ptx.cuh"
+#include "tc.cuh"
+
+namespace fairy2i {
+
+namespace pfl {
+
+constexpr int kThreads = 11 * 32;
+constexpr int kIssWarp = 8;                       // warps 8, 9: sigma / tau issuers
+constexpr int kCopyWarp = 10;
+constexpr int kTok = 64;                          // tokens per tile
+constexpr int kSteps = 16;                        // TMEM A ring: steps of 16 codes
+constexpr int kPairs = kSteps / 2;                // in pairs of steps
+constexpr int kColD = 0;                          // sigma accumulator: columns 0-127, tau 128-255
+constexpr int kColA = 256;                        // A ring: 16 columns per step (sigma, tau)
+constexpr int kTmemCols = 512;
+constexpr int kXStage = 2 * kTok * 128;           // x of 64 codes: 2 parts x 64 tokens x 128 B
+constexpr int kXS = 6;                            // x stages (also keeps one CTA per SM)
+constexpr int kCChunks = 2;                       // 128-code chunks per code stage
+constexpr int kCS = 3;                            // code stages
+constexpr int kCStage = kCChunks * 8 * 512;       // <= 8 tiles x kCChunks x 512 B
+constexpr uint64_t kWaitNs = 1000000000ull;
+// kind::f16, bf16 A and B (format 1), f32 D, K-major, N = 128, M = 128.
+constexpr uint32_t kIdesc =
+    (1u << 4) | (1u << 7) | (1u << 10) | ((128u >> 3) << 17) | ((128u >> 4) << 24);
+
+constexpr int kOffX = 0;                                        // 1024-aligned (swizzle 128 B)
+constexpr int kOffCodes = kOffX + kXS * kXStage;                // 64 KB
+constexpr int kOffRed = kOffCodes + kCS * kCStage;              // + 24 KB
+constexpr int kOffBar = kOffRed + 2 * 16 * 2 * 128 * 4;         // float [set][16 tokens][2][128]
+constexpr int kNumBars = 2 * kXS + 2 * kCS + 2 * kPairs + 6;
+constexpr int kOffMisc = kOffBar + kNumBars * 8;
+constexpr int kSmemBytes = kOffMisc + 64 + 1024;
+constexpr int kWordsPerStage = 8 * kCChunks;      // code words (steps of 16 codes) per code stage
+static_assert(kSmemBytes > 116 * 1024, "one CTA per SM: it owns all TMEM columns");
+
+struct Args {
+  const uint32_t* codes;
+  const float* scales;
+  float* y;
+  unsigned int* status;
+  int64_t B, n, out_features, ldy;
+  int wpr;          // code words per row (steps of 16 codes)
+  int nch;          // 128-code chunks per row
+  int row_tiles;    // ceil(n / 16)
+  int row_blocks;   // ceil(n / R)
+  int tok_tiles;    // ceil(B / 64)
+};
+
+// Shared-memory descriptor of a K-major operand in the 128-byte swizzle layout: rows of 128 B
+// (64 bf16 of K), 8-row groups 1024 B apart; start address advanced by 32 B per 16-element step.
+__device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t addr) {
+  return (uint64_t)((addr >> 4) & 0x3FFFu) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
+         (1ull << 46) | (2ull << 61);
+}
+
+__device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
+                                            uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %3, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %4, p;\n}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(accumulate), "r"(kIdesc)
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&v)[8]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"r"(taddr),
+      "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7])
+      : "memory");
+}
+
+// bf16 +-1 pairs of one sign plane of a code word: p holds the plane's even-code bits in byte 1
+// and odd-code bits in byte 3; register c = (code 2c, code 2c+1), 1 - 2 bit each.
+__device__ __forceinline__ void plane_bf16(uint32_t p, uint32_t (&r)[8]) {
+#pragma unroll
+  for (int c = 0; c < 8; ++c) r[c] = lop3_and_or(p << (7 - c), 0x80008000u, 0x3F803F80u);
+}
+
+__device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort,
+                                              unsigned int* status) {
+  if (*abort) return false;
+  if (mbar_wait_timed(bar, parity, kWaitNs)) return true;
+  *abort = 1;
+  latch_status(status, kStatusTimeout);
+  return false;
+}
+
+template <int T>
+__global__ void __launch_bounds__(kThreads, 1)
+    wl_prefill_kernel(const Args a, const __grid_constant__ CUtensorMap xre,
+                      const __grid_constant__ CUtensorMap xim) {
+  constexpr int TM = 2 * T;
+  constexpr int R = (T == 1) ? 64 : (T == 2 ? 32 : 16);
+  constexpr int RT = R / 16;
+  extern __shared__ unsigned char smem_raw[];
+  unsigned char* smem = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kOffBar);
+  uint64_t* xfull = bars;                   // x stage landed            (tx)
+  uint64_t* xempty = xfull + kXS;           // x stage consumed          (2 issuer commits)
+  uint64_t* cfull = xempty + kXS;           // code stage landed         (tx)
+  uint64_t* cempty = cfull + kCS;           // code stage read           (8 decoder warps)
+  uint64_t* afull = cempty + kCS;           // A step pair written       (4 warps of a set)
+  uint64_t* aempty = afull + kPairs;        // A step pair consumed      (2 issuer commits)
+  uint64_t* accf = aempty + kPairs;         // tile accumulators final   (2 issuer commits)
+  uint64_t* dempty = accf + 1;              // accumulators read out     (8 decoder warps)
+  uint64_t* fin = dempty + 1;               // [2] issued MMAs complete (end of kernel)
+  uint64_t* ebar = fin + 2;                 // [2] epilogue barrier of a decoder set (128 threads)
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + kOffMisc);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kOffMisc + 8);
+  float* red = reinterpret_cast<float*>(smem + kOffRed);
+
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int ntiles = a.row_blocks * a.tok_tiles;
+  const int my_tiles = ntiles > (int)blockIdx.x ? (ntiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
+  const int xstages = a.wpr / 4;                            // x stages (64 codes) per tile
+
+  if (tid == 0) {
+    for (int i = 0; i < kXS; ++i) {
+      mbar_init(&xfull[i], 1);
+      mbar_init(&xempty[i], 2);
+    }
+    for (int i = 0; i < kCS; ++i) {
+      mbar_init(&cfull[i], 1);
+      mbar_init(&cempty[i], 8);
+    }
+    for (int i = 0; i < kPairs; ++i) {
+      mbar_init(&afull[i], 4);
+      mbar_init(&aempty[i], 2);
+    }
+    mbar_init(accf, 2);
+    mbar_init(dempty, 8);
+    mbar_init(&fin[0], 1);
+    mbar_init(&fin[1], 1);
+    mbar_init(&ebar[0], 128);
+    mbar_init(&ebar[1], 128);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0) tmem_alloc(tmem_slot, kTmemCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  pdl_launch_dependents();
+
+  if (warp == kCopyWarp) {
+    // ---------------- producer: codes (bulk copies) and x (TMA), in K order ----------------
+    if (lane == 0) {
+      prefetch_tensormap(&xre);
+      prefetch_tensormap(&xim);
+    }
+    pdl_wait_primary();   // x may be written by the previous kernel
+    int xq = 0, cq = 0;   // running stage counters over all tiles of this CTA
+    for (int it = 0; it < my_tiles && !__shfl_sync(0xffffffffu, *abort_flag, 0); ++it) {
+      const int tile = (int)blockIdx.x + it * (int)gridDim.x;
+      const int rb = tile % a.row_blocks, tb = tile / a.row_blocks;
+      int ntl = 0;
+#pragma unroll
+      for (int rt = 0; rt < RT; ++rt) ntl += (rb * RT + rt < a.row_tiles) ? 1 : 0;
+      for (int xs = 0; xs < xstages; ++xs, ++xq) {
+        // code stage g holds chunks kCChunks g .. (kWordsPerStage steps = kWordsPerStage / 4 x stages)
+        if (xs % (kWordsPerStage / 4) == 0) {
+          const int g = xs / (kWordsPerStage / 4), st = cq % kCS;
+          const int nc = min(kCChunks, a.nch - g * kCChunks);
+          bool ok = cq < kCS ||
+                    lane != 0 || wait_or_abort(&cempty[st], ((cq / kCS) - 1) & 1, abort_flag, a.status);
+          if (!__all_sync(0xffffffffu, ok)) break;
+          if (lane == 0) mbar_arrive_expect_tx(&cfull[st], (uint32_t)(TM * ntl * nc * 512));
+          __syncwarp();
+          const int tm = lane / RT, rt = lane % RT;
+          if (lane < TM * RT && rt < ntl) {
+            const int64_t t16 = (int64_t)tm * a.row_tiles + rb * RT + rt;
+            bulk_load(smem + kOffCodes + st * kCStage + lane * kCChunks * 512,
+                      a.codes + (t16 * a.nch + g * kCChunks) * 128, (uint32_t)(nc * 512),
+                      &cfull[st]);
+          }
+          ++cq;
+        }
+        const int xst = xq % kXS;
+        bool okx = true;
+        if (lane == 0 && xq >= kXS)
+          okx = wait_or_abort(&xempty[xst], ((xq / kXS) - 1) & 1, abort_flag, a.status);
+        if (!__shfl_sync(0xffffffffu, okx, 0)) break;
+        if (lane == 0) {
+          mbar_arrive_expect_tx(&xfull[xst], (uint32_t)kXStage);
+          unsigned char* dst = smem + kOffX + xst * kXStage;
+          tma_load_2d(dst, &xre, xs * 64, tb * kTok, &xfull[xst]);
+          tma_load_2d(dst + kTok * 128, &xim, xs * 64, tb * kTok, &xfull[xst]);
+        }
+        __syncwarp();
+      }
+    }
+    // Copies still in flight (after an abort) land before the CTA exits: wait for the last phase
+    // of every stage that was filled.
+    if (lane == 0) {
+      for (int q = max(0, xq - kXS); q < xq; ++q)
+        (void)mbar_wait_timed(&xfull[q % kXS], (q / kXS) & 1, kWaitNs);
+      for (int q = max(0, cq - kCS); q < cq; ++q)
+        (void)mbar_wait_timed(&cfull[q % kCS], (q / kCS) & 1, kWaitNs);
+    }
+    __syncwarp();
+  } else if (warp == kIssWarp || warp == kIssWarp + 1) {
+    // ---------------- MMA issuers: warp 8 the sigma plane, warp 9 the tau plane ----------------
+    const int e = warp - kIssWarp;
+    if (lane == 0) {
+      int p = 0, xq = 0;
+      const int npt = a.wpr / 2;   // step pairs per tile (a tile has 4 steps per x stage)
+      for (int it = 0; it < my_tiles; ++it) {
+        if (it > 0 && !wait_or_abort(dempty, (it - 1) & 1, abort_flag, a.status)) break;
+        tc_fence_after();
+        bool ok = true;
+        for (int pp = 0; pp < npt && ok; ++pp, ++p) {
+          const int xst = xq % kXS;
+          if ((pp & 1) == 0) ok = wait_or_abort(&xfull[xst], (xq / kXS) & 1, abort_flag, a.status);
+          ok = ok && wait_or_abort(&afull[p % kPairs], (p / kPairs) & 1, abort_flag, a.status);
+          if (!ok) break;
+          tc_fence_after();
+          const uint32_t xaddr = smem_u32(smem + kOffX + xst * kXStage) + (pp & 1) * 64;
+          const uint32_t acol = tmem + kColA + (p % kPairs) * 32 + e * 8;
+          mma_bf16_ts(tmem + kColD + e * 128, acol, smem_desc_sw128(xaddr), pp > 0 ? 1u : 0u);
+          mma_bf16_ts(tmem + kColD + e * 128, acol + 16, smem_desc_sw128(xaddr + 32), 1u);
+          mma_commit(&aempty[p % kPairs]);
+          if (pp & 1) {
+            mma_commit(&xempty[xst]);
+            ++xq;
+          }
+        }
+        if (!ok) break;
+        mma_commit(accf);
+      }
+      // Every MMA this thread issued completes before TMEM is released.
+      mma_commit(&fin[e]);
+      (void)mbar_wait_timed(&fin[e], 0, kWaitNs);
+    }
+    __syncwarp();
+  } else {
+    // ---------------- warps 0-7: decode + epilogue ----------------
+    const int set = warp >> 2, quarter = warp & 3, L = quarter * 32 + lane;
+    const uint32_t t_lane = tmem + ((uint32_t)(quarter * 32) << 16);
+    const int tl = L >> 4, rl = L & 15;   // 16-row tile (tm * RT + rt) and row within it
+    const int npt = a.wpr / 2;            // step pairs per tile
+    constexpr int kPairsPerStage = kWordsPerStage / 2;
+    float* sred = red + set * (16 * 2 * 128);
+    int cq0 = 0;                          // code stages of the earlier tiles
+    uint32_t eph = 0;                     // phases of this set's epilogue barrier passed
+    // Barrier of the set's 128 threads with a bounded wait (false: the kernel aborts).
+    auto set_sync = [&]() -> bool {
+      mbar_arrive(&ebar[set]);
+      const bool ok = mbar_wait_timed(&ebar[set], eph & 1, kWaitNs);
+      ++eph;
+      if (!__all_sync(0xffffffffu, ok)) {
+        *abort_flag = 1;
+        if (lane == 0) latch_status(a.status, kStatusTimeout);
+        return false;
+      }
+      return true;
+    };
+    for (int it = 0; it < my_tiles; ++it) {
+      const int tile = (int)blockIdx.x + it * (int)gridDim.x;
+      const int rb = tile % a.row_blocks, tb = tile / a.row_blocks;
+      const int nstages = (npt + kPairsPerStage - 1) / kPairsPerStage;
+      bool ok = true;
+      for (int pp = set; pp < npt && ok; pp += 2) {
+        const int p = it * npt + pp;
+        const int g = pp / kPairsPerStage, cq = cq0 + g, st = cq % kCS;
+        ok = __all_sync(0xffffffffu, wait_or_abort(&cfull[st], (cq / kCS) & 1, abort_flag, a.status));
+        if (ok && p >= kPairs)
+          ok = __all_sync(0xffffffffu, wait_or_abort(&aempty[p % kPairs], ((p / kPairs) - 1) & 1,
+                                                     abort_flag, a.status));
+        if (!ok) break;
+        const int wi = (pp % kPairsPerStage) * 2;   // first word of the pair in the stage
+        const uint2 w2 = *reinterpret_cast<const uint2*>(
+            smem + kOffCodes + st * kCStage + (tl * kCChunks + (wi >> 3)) * 512 + rl * 32 +
+            (wi & 7) * 4);
+        uint32_t r[32];
+        uint32_t* rp = r;
+        plane_bf16(prmt(w2.x, 0u, 0x1404u), *reinterpret_cast<uint32_t(*)[8]>(rp));       // sigma, step 2pp
+        plane_bf16(prmt(w2.x, 0u, 0x3424u), *reinterpret_cast<uint32_t(*)[8]>(rp + 8));   // tau
+        plane_bf16(prmt(w2.y, 0u, 0x1404u), *reinterpret_cast<uint32_t(*)[8]>(rp + 16));  // sigma, 2pp+1
+        plane_bf16(prmt(w2.y, 0u, 0x3424u), *reinterpret_cast<uint32_t(*)[8]>(rp + 24));  // tau
+        const bool last_in_stage =
+            pp + 2 >= min((g + 1) * kPairsPerStage, npt);   // this set's last pair of the stage
+        __syncwarp();
+        if (lane == 0 && last_in_stage) mbar_arrive(&cempty[st]);
+        tmem_st32(t_lane + kColA + (p % kPairs) * 32, r);
+        tmem_wait_st();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&afull[p % kPairs]);
+      }
+      cq0 += nstages;
+      if (!ok) break;
+
+      // ---- epilogue of the tile: set s takes tokens 32 s .. 32 s + 31, in blocks of 16 ----
+      ok = __all_sync(0xffffffffu, wait_or_abort(accf, it & 1, abort_flag, a.status));
+      if (!ok) break;
+      tc_fence_after();
+      const int tm = L / R;
+      const bool valid = L < TM * R;
+      const int t = tm >> 1, mat = tm & 1;
+      const float hr = valid ? 0.5f * __ldg(a.scales + (t * 2 + mat) * 2 + 0) : 0.f;
+      const float hi = valid ? 0.5f * __ldg(a.scales + (t * 2 + mat) * 2 + 1) : 0.f;
+      for (int sb2 = 0; sb2 < 2; ++sb2) {
+        const int sb = set * 2 + sb2;
+        float pr[16], pi[16], qr[16], qi[16];
+        tmem_ld16(t_lane + kColD + sb * 16, pr);
+        tmem_ld16(t_lane + kColD + 64 + sb * 16, pi);
+        tmem_ld16(t_lane + kColD + 128 + sb * 16, qr);
+        tmem_ld16(t_lane + kColD + 192 + sb * 16, qi);
+        tmem_wait_ld();
+        if (sb2 == 1) {
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(dempty);   // the issuers may start the next tile
+        }
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+          float Pr = pr[k], Pi = pi[k], Qr = qr[k], Qi = qi[k];
+          if (mat) {                 // W multiplies conj(x)
+            Pi = -Pi;
+            Qi = -Qi;
+          }
+          sred[(k * 2 + 0) * 128 + L] = valid ? hr * Pr - hi * Pi + hr * Qr + hi * Qi : 0.f;
+          sred[(k * 2 + 1) * 128 + L] = valid ? hr * Pi + hi * Pr + hr * Qi - hi * Qr : 0.f;
+        }
+        if (!set_sync()) break;
+        // sum over the stage-matrices; item = (token k, part, row r)
+        for (int item = L; item < 16 * 2 * R; item += 128) {
+          const int rr = item % R, kp = item / R;
+          float sum = 0.f;
+#pragma unroll
+          for (int m2 = 0; m2 < TM; ++m2) sum += sred[kp * 128 + m2 * R + rr];
+          const int64_t b = (int64_t)tb * kTok + sb * 16 + (kp >> 1);
+          const int64_t j = (int64_t)rb * R + rr;
+          if (b < a.B && j < a.n) {
+            if ((kp & 1) == 0) a.y[b * a.ldy + j] = sum;
+            else if (a.n + j < a.out_features) a.y[b * a.ldy + a.n + j] = sum;
+          }
+        }
+        if (!set_sync()) break;
+      }
+      if (__shfl_sync(0xffffffffu, *abort_flag, 0)) break;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 0) tmem_dealloc(tmem, kTmemCols);
+}
+
+template <int T>
+fairy2i_status launch(const Args& a, const CUtensorMap& xre, const CUtensorMap& xim, int grid,
+                      cudaStream_t stream) {
+  auto kern = wl_prefill_kernel<T>;
+  static bool configured = false;
+  if (!configured) {
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) !=
+        cudaSuccess)
+      return FAIRY2I_ERR_CUDA;
+    configured = true;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (cudaLaunchKernelEx(&cfg, kern, a, xre, xim) != cudaSuccess) return FAIRY2I_ERR_CUDA;
+  return FAIRY2I_OK;
+}
+
+}  // namespace pfl
+
+namespace {
+std::mutex g_pfl_mu;
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+int g_pfl_sms[64];
+}  // namespace
+
+static PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  std::lock_guard<std::mutex> lock(g_pfl_mu);
+  if (!g_encode) {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                         &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      return nullptr;
+    g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  }
+  return g_encode;
+}
+
+// 2-D map over one part of x: `width` bf16 values per token row (zero beyond), rows `ldx` apart,
+// B rows; box of 64 values x 64 tokens, 128-byte swizzle.
+static bool encode_x_map(CUtensorMap* map, const void* base, int64_t width, int64_t B,
+                         int64_t ldx) {
+  PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
+  if (!enc || width < 1) return false;
+  const cuuint64_t dims[2] = {(cuuint64_t)width, (cuuint64_t)B};
+  const cuuint64_t strides[1] = {(cuuint64_t)ldx * 2};
+  const cuuint32_t box[2] = {64, (cuuint32_t)pfl::kTok};
+  const cuuint32_t estr[2] = {1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Handles bf16 x with 16-byte aligned rows (ldx % 8 == 0), m % 8 == 0 and T <= 4; anything else
+// is left to the other kernels (*handled = false).
+fairy2i_status launch_wl_prefill(const void* x, fairy2i_dtype xdt, int64_t B, int64_t in_features,
+                                 int64_t ldx, const uint32_t* codes, const float* scales,
+                                 int64_t n, int64_t m, int64_t out_features, int64_t wpr, int T,
+                                 float* y, int64_t ldy, cudaStream_t stream, bool* handled) {
+  using namespace pfl;
+  *handled = false;
+  if (xdt != FAIRY2I_BF16 || T > 4 || (reinterpret_cast<uintptr_t>(x) % 16) != 0 ||
+      ldx % 8 != 0 || m % 8 != 0 || B > (int64_t(1) << 30) || wpr > (int64_t(1) << 24))
+    return FAIRY2I_OK;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return FAIRY2I_ERR_CUDA;
+  {
+    std::lock_guard<std::mutex> lock(g_pfl_mu);
+    if (!g_pfl_sms[dev] &&
+        cudaDeviceGetAttribute(&g_pfl_sms[dev], cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return FAIRY2I_ERR_CUDA;
+  }
+  CUtensorMap xre, xim;
+  const __nv_bfloat16* xb = reinterpret_cast<const __nv_bfloat16*>(x);
+  if (!encode_x_map(&xre, xb, m, B, ldx)) return FAIRY2I_OK;
+  const bool has_im = in_features > m;
+  if (!encode_x_map(&xim, has_im ? xb + m : xb, has_im ? in_features - m : 1, B, ldx))
+    return FAIRY2I_OK;
+  const int R = T == 1 ? 64 : (T == 2 ? 32 : 16);
+  Args a;
+  a.codes = codes;
+  a.scales = scales;
+  a.y = y;
+  a.status = device_status_word();
+  a.B = B; a.n = n; a.out_features = out_features; a.ldy = ldy;
+  a.wpr = (int)wpr; a.nch = (int)(wpr / 8); a.row_tiles = (int)((n + 15) / 16);
+  a.row_blocks = (int)((n + R - 1) / R);
+  a.tok_tiles = (int)((B + kTok - 1) / kTok);
+  const int64_t tiles = (int64_t)a.row_blocks * a.tok_tiles;
+  if (tiles > (int64_t(1) << 30)) return FAIRY2I_OK;
+  const int grid = (int)(tiles < g_pfl_sms[dev] ? tiles : g_pfl_sms[dev]);
+  *handled = true;
+  switch (T) {
+    case 1: return launch<1>(a, xre, xim, grid, stream);
+    case 2: return launch<2>(a, xre, xim, grid, stream);
+    case 3: return launch<3>(a, xre, xim, grid, stream);
+    case 4: return launch<4>(a, xre, xim, grid, stream);
+  }
+  *handled = false;
+  return FAIRY2I_OK;
+}
+
+}  // namespace fairy2i

@@ -89,7 +89,7 @@ def test_wl_matmul_validation(lib):
         return lib.fairy2i_wl_matmul_path(x, xdt, B, inf, ldx, codes, scales, outf, T, y, ldy,
                                           path, None)
     assert call(B=0) == 0                      # empty batch: nothing to do
-    assert call(B=-1) == 1 and call(T=0) == 1 and call(path=3) == 1 and call(x=None) == 1
+    assert call(B=-1) == 1 and call(T=0) == 1 and call(path=4) == 1 and call(x=None) == 1
     assert call(xdt=7) == 4
     assert call(ldx=15) == 2 and call(ldy=15) == 2
     assert call(x=ODD) == 3 and call(codes=ODD) == 3

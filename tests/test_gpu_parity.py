@@ -227,9 +227,10 @@ def test_wl_matmul_full_size_decode(F, rows, cols, B, seed):
     assert_wl_close(yg, yo, xo, so)
 
 
-@pytest.mark.parametrize("rows,cols,T", [(11008, 4096, 1), (4096, 11008, 3)])
+@pytest.mark.parametrize("rows,cols,T", [(11008, 4096, 1), (11008, 4096, 2), (4096, 11008, 3)])
 def test_wl_matmul_prefill_sampled(F, rows, cols, T):
-    """2048 tokens; the oracle computes a sample of 96 output rows for every token."""
+    """2048 tokens through the default path (the tcgen05 prefill GEMM); the oracle computes a
+    sample of 96 output rows for every token."""
     seed = synth.weight_seed("prefill", 0 if rows > cols else 1)
     co, so = _layer(rows, cols, T, seed)
     B = 2048
@@ -333,3 +334,88 @@ def test_wl_tcgen05_rejects_outside_its_domain(F):
         with pytest.raises(F.Fairy2iError) as e:
             F.wl_matmul(x, cd, sc, 2 * n, path=2)
         assert e.value.code == 1
+
+
+# ------------------------------------------------------------------------------ tcgen05 prefill
+@pytest.mark.parametrize("out_f,in_f,T,B", [
+    (64, 256, 1, 64), (64, 256, 2, 3), (37, 144, 2, 70), (64, 256, 3, 130), (64, 256, 4, 64),
+    (50, 272, 4, 9), (2, 16, 1, 5), (4096, 4096, 2, 64), (256, 2048, 2, 130), (96, 1024, 3, 200),
+    (1000, 4096, 2, 65), (130, 400, 1, 129),
+])
+def test_wl_tcgen05_prefill_path(F, out_f, in_f, T, B):
+    """The tcgen05 prefill GEMM (path 3): ragged row blocks (R = 64, 32, 16, 16 rows of every
+    stage-matrix for T = 1..4), ragged token tiles (64 tokens), ragged 64-code x stages and
+    128-code chunks, one CTA or many tiles per CTA."""
+    n, m = O.complex_dims(out_f, in_f)
+    codes, scales = _random_quantized(n, m, T, seed=5 * out_f + 3 * in_f + T)
+    x = synth.outlier_activations(B, in_f, seed=out_f + in_f + 2)
+    yg = _run_wl(F, x, codes, scales, out_f, path=3)
+    xo = x.float().numpy()
+    assert_wl_close(yg, O.wl_matmul(xo, codes, scales, out_f), xo, scales)
+
+
+@pytest.mark.parametrize("T", [1, 2, 3, 4])
+def test_wl_tcgen05_prefill_all_codes_each_value(F, T):
+    """Every code value at every word position of every stage-matrix lane block, 70 tokens."""
+    n, m = 40, 384
+    codes = np.zeros((T, 2, n, m), dtype=np.uint8)
+    for t in range(T):
+        for j in range(n):
+            codes[t, 0, j] = (np.arange(m) + j + t) % 4
+            codes[t, 1, j] = (np.arange(m) // 16 + 3 * j + t) % 4
+    g = np.random.default_rng(10 + T)
+    scales = (0.01 + 0.02 * g.random((T, 2, 2))).astype(np.float32)
+    x = synth.outlier_activations(70, 2 * m, seed=17 + T)
+    yg = _run_wl(F, x, codes, scales, 2 * n, path=3)
+    xo = x.float().numpy()
+    assert_wl_close(yg, O.wl_matmul(xo, codes, scales, 2 * n), xo, scales)
+
+
+def test_wl_tcgen05_prefill_strided_odd_input(F):
+    """Odd in_features (the last Im channel padded) read through a row stride that keeps rows
+    16-byte aligned; y written into a wider buffer."""
+    m, T, B = 72, 2, 77
+    in_f, n = 2 * m - 1, 45
+    codes, scales = _random_quantized(n, m, T, seed=21)
+    xbig = synth.outlier_activations(B, 152, seed=22)
+    x = xbig.to(DEV)[:, :in_f]
+    y = torch.full((B, 2 * n + 8), 7.0, device=DEV)
+    F.wl_matmul(x, upload_codes(O.pack_codes(codes)), torch.from_numpy(scales).to(DEV), 2 * n,
+                y=y[:, : 2 * n], path=3)
+    assert F.get_status() == 0
+    yg = y.cpu().numpy()
+    assert np.all(yg[:, 2 * n:] == 7.0)
+    xo = xbig[:, :in_f].float().numpy()
+    assert_wl_close(yg[:, : 2 * n], O.wl_matmul(xo, codes, scales, 2 * n), xo, scales)
+
+
+def test_wl_auto_path_routes_batches_to_prefill(F):
+    """Above two tokens the default path is the prefill GEMM where it applies: same bits."""
+    n, m, T, B = 300, 512, 2, 33
+    codes, scales = _random_quantized(n, m, T, seed=23)
+    cd = upload_codes(O.pack_codes(codes))
+    sc = torch.from_numpy(scales).to(DEV)
+    x = synth.outlier_activations(B, 2 * m, seed=24).to(DEV)
+    y0 = F.wl_matmul(x, cd, sc, 2 * n, path=0)
+    y3 = F.wl_matmul(x, cd, sc, 2 * n, path=3)
+    assert F.get_status() == 0
+    assert torch.equal(y0, y3)
+
+
+def test_wl_tcgen05_prefill_rejects_outside_its_domain(F):
+    n, m, T = 16, 64, 2
+    codes, scales = _random_quantized(n, m, T, seed=25)
+    cd = upload_codes(O.pack_codes(codes))
+    sc = torch.from_numpy(scales).to(DEV)
+    xs = [torch.zeros((8, 2 * m), dtype=torch.float32, device=DEV),                    # fp32 x
+          synth.outlier_activations(8, 2 * m - 1, seed=2).to(DEV)]                     # ldx = 127
+    for x in xs:
+        with pytest.raises(F.Fairy2iError) as e:
+            F.wl_matmul(x, cd, sc, 2 * n, path=3)
+        assert e.value.code == 1
+    codes5, scales5 = _random_quantized(n, m, 5, seed=26)                              # T = 5
+    with pytest.raises(F.Fairy2iError) as e:
+        F.wl_matmul(synth.outlier_activations(8, 2 * m, seed=3).to(DEV),
+                    upload_codes(O.pack_codes(codes5)), torch.from_numpy(scales5).to(DEV),
+                    2 * n, path=3)
+    assert e.value.code == 1
