@@ -7,6 +7,11 @@ quantized linears. Metric: decode GB/s = algorithmic bytes (packed codes + scale
 every linear) per second, against the HBM copy peak. The 1.62 GB of codes per step exceed the
 L2 many times over, so no L2 flush is needed between steps.
 
+The line also carries a "prefill" object: the tensor-core GEMM path on 2048 tokens through the
+4096 -> 11008 and 11008 -> 4096 layers at T = 1, 2, 3 (effective TOPS = 8 n m B / time, and the
+MMA work 16 T n m B / time against the bf16 tensor peak), each launch timed alone with CUDA
+events after an L2 flush.
+
 --impl reference times the CPU oracle (float64 numpy) on the host cores on a bounded sample of
 the same workload and reports the same metric.
 
@@ -44,6 +49,10 @@ def peaks():
         return float(p["hbm_gbs"]), float(p["bf16_tflops"]), "measured"
     except Exception:
         return 6800.0, 1900.0, "fallback"
+
+
+PREFILL_TOKENS = 2048
+PREFILL_LAYERS = (("up", 11008, 4096, 0), ("down", 4096, 11008, 1))   # (name, out, in, seed idx)
 
 
 def layer_shapes(layers: int):
@@ -215,8 +224,9 @@ def run_ours(args, world, rank, local):
     ms = max_over_ranks(ms, world)
     ms_step = ms / args.steps
     value = world * step_bytes * args.steps / (ms * 1e-3) / 1e9
-    if F.get_status() != 0:
-        raise RuntimeError("device status after timed region")
+    st = F.get_status()
+    if st != 0:
+        raise RuntimeError(f"device status {st} after the timed region")
 
     # end to end through the public call with host buffers: per step the inputs of all
     # linears go host->device from pinned memory and every output comes back to the host.
@@ -247,6 +257,9 @@ def run_ours(args, world, rank, local):
         e3.record(stream)
     stream.synchronize()
     ms_e2e = max_over_ranks(e2.elapsed_time(e3), world)
+    st = F.get_status()
+    if st != 0:
+        raise RuntimeError(f"device status {st} after the end-to-end steps")
     e2e_value = world * step_bytes * e2e_steps / (ms_e2e * 1e-3) / 1e9
 
     hbm, _, peak_kind = peaks()
@@ -271,9 +284,74 @@ def run_ours(args, world, rank, local):
                      "kernel": "wl_matmul decode (all launches of the step)"},
         "clocks": clk,
     }
+    if not args.no_prefill:
+        del stack
+        torch.cuda.empty_cache()
+        line["prefill"] = run_prefill(F, dev, args.prefill_steps, max(args.warmup, 3))
     if rank == 0 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(B, budget_s=args.cpu_budget)
     return line
+
+
+def run_prefill(F, dev, steps: int, warmup: int):
+    """Prefill GEMM on 2048 tokens: per layer and T, the median over `steps` launches, each timed
+    alone (CUDA events on the launching stream) after a 256 MB L2 flush."""
+    _, bf16, peak_kind = peaks()
+    stream = torch.cuda.Stream(device=dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    rows_out, roof = [], None
+    clocks = Clocks(torch.cuda.current_device())
+    clocks.start()
+    for (name, rows, cols, idx) in PREFILL_LAYERS:
+        seed = synth.weight_seed("prefill", idx)
+        R = synth.student_t_weight(rows, cols, seed, device=dev)
+        U, W = F.convert(R)
+        del R
+        codes, scales = F.quantize(U, W, 3)     # stages 0..T-1 of a T = 3 quantization are the
+        del U, W                                # T-stage quantization (prefix of the buffers)
+        x = synth.outlier_activations(PREFILL_TOKENS, cols,
+                                      synth.activation_seed(seed, PREFILL_TOKENS), device=dev)
+        y = torch.empty((PREFILL_TOKENS, rows), dtype=torch.float32, device=dev)
+        n, m = (rows + 1) // 2, (cols + 1) // 2
+        # The set-up ran on the current stream (and y may reuse the blocks of U, W): the timed
+        # launches on `stream` start after it.
+        stream.wait_stream(torch.cuda.current_stream())
+        for T in (1, 2, 3):
+            times = []
+            with torch.cuda.stream(stream):
+                for i in range(warmup + steps):
+                    flush.zero_()
+                    e0 = torch.cuda.Event(enable_timing=True)
+                    e1 = torch.cuda.Event(enable_timing=True)
+                    e0.record(stream)
+                    F.wl_matmul(x, codes, scales, rows, y=y, stream=stream, T=T)
+                    e1.record(stream)
+                    if i >= warmup:
+                        times.append((e0, e1))
+            stream.synchronize()
+            st = F.get_status()
+            if st != 0:
+                raise RuntimeError(f"device status {st} after the prefill launches")
+            us = statistics.median(a.elapsed_time(b) for a, b in times) * 1e3
+            eff = 8.0 * n * m * PREFILL_TOKENS / (us * 1e-6) / 1e12
+            mma = 2 * T * eff
+            rows_out.append({"layer": f"{name} {cols}->{rows}", "T": T, "us": round(us, 1),
+                             "effective_tops": round(eff, 1), "mma_tflops": round(mma, 1),
+                             "tensor_frac": round(mma / bf16, 4)})
+            if name == "up" and T == T_STAGES:
+                roof = {"bound": "tensor", "achieved": round(mma, 1), "peak": bf16,
+                        "unit": "TFLOP/s", "frac": round(mma / bf16, 4), "traffic": None,
+                        "peak_kind": f"{peak_kind} bf16_tflops (burst)",
+                        "kernel": f"wl_prefill_kernel<{T}> (up {cols}->{rows}, "
+                                  f"{PREFILL_TOKENS} tokens)"}
+        del codes, scales, x, y
+    clk = clocks.stop()
+    del flush
+    return {"workload": f"prefill {PREFILL_TOKENS} tokens x (4096->11008, 11008->4096), bf16 x",
+            "metric": "effective TOPS = 8 n m B / time; MMA work 16 T n m B / time",
+            "timing": "median of per-launch CUDA-event times, L2 flushed before each launch",
+            "layers": rows_out, "roofline": roof, "clocks": clk,
+            "gpu_launches": len(rows_out) * steps}
 
 
 # --------------------------------------------------------------------------------------------
@@ -366,6 +444,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--ref-linears", type=int, default=2)
+    ap.add_argument("--no-prefill", action="store_true")
+    ap.add_argument("--prefill-steps", type=int, default=10)
     args = ap.parse_args()
     world, rank, local = dist_setup()
     if args.impl == "reference":

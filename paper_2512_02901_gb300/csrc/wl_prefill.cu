@@ -12,16 +12,24 @@
 // kind::f16 (M = 128, N = 128, K = 16) run: A = the sigma (or tau) plane of the word as bf16 +-1 in
 // tensor memory, B = x of the 64 tokens (rows 0-63: Re x, rows 64-127: Im x) in shared memory, D =
 // the sigma accumulator (TMEM columns 0-127) or the tau accumulator (128-255): column p*64 + b is
-// the sum for part p (re/im) of token b. x arrives by TMA (128-byte swizzle, one box of 64 codes x
+// the sum for part p (re/im) of token b. x arrives by TMA (128-byte swizzle, boxes of 64 codes x
 // 64 tokens per part; Re and Im through two tensor maps so that each part is zero beyond its end).
 // The CTAs are persistent over the tiles, ordered token-tile-major so that CTAs running together
 // share x in L2.
 //
+// Pipeline granularity: a group = 64 codes = 4 steps of 16 codes = 2 step pairs. The A ring holds
+// 4 groups (64 TMEM columns each); an x stage holds 128 codes (two groups). Per group an issuer
+// makes one barrier wait (the group's full barrier, which the decoders complete once the A pairs
+// are stored and x has landed) and one commit (plus one per x stage): the issue cost per MMA is
+// what bounds this kernel once the waits are per MMA.
+//
 // Roles (11 warps): warps 0-7, two sets of four (warp w reaches TMEM lanes 32 (w % 4) ..), decode
-// the code words into the TMEM A ring, set s taking the step pairs p = s (mod 2) (one 32-column
-// store per pair: sigma, tau of two steps of 16 codes), and run the epilogue of each tile, set s for
-// tokens 32 s .. 32 s + 31; warps 8 and 9 issue the sigma and the tau MMAs (one commit per pair
-// each); warp 10 copies the codes (bulk copies of whole 16-row tiles) and x (TMA) in.
+// the code words into the A ring, set s taking pair s of every group (one 32-column store: sigma,
+// tau of two steps), warp 0 also relaying the x-stage arrival into the group barrier; then they run
+// the epilogue of each tile, set s for tokens 32 s .. 32 s + 31 (all accumulator columns are read
+// out first, so the MMAs of the next tile start before the reduction and the stores). Warps 8 and
+// 9 issue the sigma and the tau MMAs; warp 10 copies the codes (bulk copies of whole 16-row tiles)
+// and x (TMA) in.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
@@ -40,30 +48,32 @@ constexpr int kThreads = 11 * 32;
 constexpr int kIssWarp = 8;                       // warps 8, 9: sigma / tau issuers
 constexpr int kCopyWarp = 10;
 constexpr int kTok = 64;                          // tokens per tile
-constexpr int kSteps = 16;                        // TMEM A ring: steps of 16 codes
-constexpr int kPairs = kSteps / 2;                // in pairs of steps
+constexpr int kG = 4;                             // A ring: groups of 64 codes (4 steps)
 constexpr int kColD = 0;                          // sigma accumulator: columns 0-127, tau 128-255
-constexpr int kColA = 256;                        // A ring: 16 columns per step (sigma, tau)
+constexpr int kColA = 256;                        // A ring: 64 columns per group
 constexpr int kTmemCols = 512;
-constexpr int kXStage = 2 * kTok * 128;           // x of 64 codes: 2 parts x 64 tokens x 128 B
-constexpr int kXS = 6;                            // x stages (also keeps one CTA per SM)
-constexpr int kCChunks = 2;                       // 128-code chunks per code stage
+constexpr int kXSub = 2 * kTok * 128;             // x of 64 codes: 2 parts x 64 tokens x 128 B
+constexpr int kXStage = 2 * kXSub;                // x stage: 128 codes
+constexpr int kXS = 4;                            // x stages
+constexpr int kCChunks = 2;                       // 128-code chunks per code stage (4 groups)
 constexpr int kCS = 3;                            // code stages
 constexpr int kCStage = kCChunks * 8 * 512;       // <= 8 tiles x kCChunks x 512 B
+constexpr int kGroupsPerCStage = 2 * kCChunks;
+constexpr int kRedSet = 2 * 16 * 2 * 128;         // floats: [sub-block][16 tokens][2][128 lanes]
 constexpr uint64_t kWaitNs = 1000000000ull;
 // kind::f16, bf16 A and B (format 1), f32 D, K-major, N = 128, M = 128.
 constexpr uint32_t kIdesc =
     (1u << 4) | (1u << 7) | (1u << 10) | ((128u >> 3) << 17) | ((128u >> 4) << 24);
 
 constexpr int kOffX = 0;                                        // 1024-aligned (swizzle 128 B)
-constexpr int kOffCodes = kOffX + kXS * kXStage;                // 64 KB
+constexpr int kOffCodes = kOffX + kXS * kXStage;                // 128 KB
 constexpr int kOffRed = kOffCodes + kCS * kCStage;              // + 24 KB
-constexpr int kOffBar = kOffRed + 2 * 16 * 2 * 128 * 4;         // float [set][16 tokens][2][128]
-constexpr int kNumBars = 2 * kXS + 2 * kCS + 2 * kPairs + 6;
+constexpr int kOffBar = kOffRed + 2 * kRedSet * 4;              // + 64 KB
+constexpr int kNumBars = 2 * kXS + 2 * kCS + 2 * kG + 6;
 constexpr int kOffMisc = kOffBar + kNumBars * 8;
 constexpr int kSmemBytes = kOffMisc + 64 + 1024;
-constexpr int kWordsPerStage = 8 * kCChunks;      // code words (steps of 16 codes) per code stage
 static_assert(kSmemBytes > 116 * 1024, "one CTA per SM: it owns all TMEM columns");
+static_assert(kSmemBytes <= 227 * 1024, "shared memory per CTA");
 
 struct Args {
   const uint32_t* codes;
@@ -72,7 +82,7 @@ struct Args {
   unsigned int* status;
   int64_t B, n, out_features, ldy;
   int wpr;          // code words per row (steps of 16 codes)
-  int nch;          // 128-code chunks per row
+  int nch;          // 128-code chunks per row (= x stages per tile)
   int row_tiles;    // ceil(n / 16)
   int row_blocks;   // ceil(n / R)
   int tok_tiles;    // ceil(B / 64)
@@ -94,22 +104,17 @@ __device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, ui
       : "memory");
 }
 
-__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&v)[8]) {
-  asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"r"(taddr),
-      "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7])
-      : "memory");
-}
-
 // bf16 +-1 pairs of one sign plane of a code word: p holds the plane's even-code bits in byte 1
 // and odd-code bits in byte 3; register c = (code 2c, code 2c+1), 1 - 2 bit each.
-__device__ __forceinline__ void plane_bf16(uint32_t p, uint32_t (&r)[8]) {
+__device__ __forceinline__ void plane_bf16(uint32_t p, uint32_t* r) {
 #pragma unroll
   for (int c = 0; c < 8; ++c) r[c] = lop3_and_or(p << (7 - c), 0x80008000u, 0x3F803F80u);
 }
 
+// Bounded wait; the first try is the fast path, the abort flag is looked at only after it fails.
 __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort,
                                               unsigned int* status) {
+  if (mbar_try_wait(bar, parity)) return true;
   if (*abort) return false;
   if (mbar_wait_timed(bar, parity, kWaitNs)) return true;
   *abort = 1;
@@ -132,9 +137,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* xempty = xfull + kXS;           // x stage consumed          (2 issuer commits)
   uint64_t* cfull = xempty + kXS;           // code stage landed         (tx)
   uint64_t* cempty = cfull + kCS;           // code stage read           (8 decoder warps)
-  uint64_t* afull = cempty + kCS;           // A step pair written       (4 warps of a set)
-  uint64_t* aempty = afull + kPairs;        // A step pair consumed      (2 issuer commits)
-  uint64_t* accf = aempty + kPairs;         // tile accumulators final   (2 issuer commits)
+  uint64_t* gfull = cempty + kCS;           // group's A stored, x in    (8 decoder warps)
+  uint64_t* gempty = gfull + kG;            // group's A consumed        (2 issuer commits)
+  uint64_t* accf = gempty + kG;             // tile accumulators final   (2 issuer commits)
   uint64_t* dempty = accf + 1;              // accumulators read out     (8 decoder warps)
   uint64_t* fin = dempty + 1;               // [2] issued MMAs complete (end of kernel)
   uint64_t* ebar = fin + 2;                 // [2] epilogue barrier of a decoder set (128 threads)
@@ -145,7 +150,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int ntiles = a.row_blocks * a.tok_tiles;
   const int my_tiles = ntiles > (int)blockIdx.x ? (ntiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
-  const int xstages = a.wpr / 4;                            // x stages (64 codes) per tile
+  const int gpt = a.wpr / 4;          // groups per tile (even: 2 per 128-code chunk)
+  const int nch = a.nch;              // x stages per tile
 
   if (tid == 0) {
     for (int i = 0; i < kXS; ++i) {
@@ -156,9 +162,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&cfull[i], 1);
       mbar_init(&cempty[i], 8);
     }
-    for (int i = 0; i < kPairs; ++i) {
-      mbar_init(&afull[i], 4);
-      mbar_init(&aempty[i], 2);
+    for (int i = 0; i < kG; ++i) {
+      mbar_init(&gfull[i], 8);
+      mbar_init(&gempty[i], 2);
     }
     mbar_init(accf, 2);
     mbar_init(dempty, 8);
@@ -190,11 +196,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       int ntl = 0;
 #pragma unroll
       for (int rt = 0; rt < RT; ++rt) ntl += (rb * RT + rt < a.row_tiles) ? 1 : 0;
-      for (int xs = 0; xs < xstages; ++xs, ++xq) {
-        // code stage g holds chunks kCChunks g .. (kWordsPerStage steps = kWordsPerStage / 4 x stages)
-        if (xs % (kWordsPerStage / 4) == 0) {
-          const int g = xs / (kWordsPerStage / 4), st = cq % kCS;
-          const int nc = min(kCChunks, a.nch - g * kCChunks);
+      for (int xs = 0; xs < nch; ++xs, ++xq) {
+        if (xs % kCChunks == 0) {   // code stage: chunks xs .. xs + kCChunks - 1
+          const int st = cq % kCS;
+          const int nc = min(kCChunks, nch - xs);
           bool ok = cq < kCS ||
                     lane != 0 || wait_or_abort(&cempty[st], ((cq / kCS) - 1) & 1, abort_flag, a.status);
           if (!__all_sync(0xffffffffu, ok)) break;
@@ -204,8 +209,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (lane < TM * RT && rt < ntl) {
             const int64_t t16 = (int64_t)tm * a.row_tiles + rb * RT + rt;
             bulk_load(smem + kOffCodes + st * kCStage + lane * kCChunks * 512,
-                      a.codes + (t16 * a.nch + g * kCChunks) * 128, (uint32_t)(nc * 512),
-                      &cfull[st]);
+                      a.codes + (t16 * a.nch + xs) * 128, (uint32_t)(nc * 512), &cfull[st]);
           }
           ++cq;
         }
@@ -217,8 +221,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) {
           mbar_arrive_expect_tx(&xfull[xst], (uint32_t)kXStage);
           unsigned char* dst = smem + kOffX + xst * kXStage;
-          tma_load_2d(dst, &xre, xs * 64, tb * kTok, &xfull[xst]);
-          tma_load_2d(dst + kTok * 128, &xim, xs * 64, tb * kTok, &xfull[xst]);
+          tma_load_2d(dst, &xre, xs * 128, tb * kTok, &xfull[xst]);
+          tma_load_2d(dst + kXSub / 2, &xim, xs * 128, tb * kTok, &xfull[xst]);
+          tma_load_2d(dst + kXSub, &xre, xs * 128 + 64, tb * kTok, &xfull[xst]);
+          tma_load_2d(dst + kXSub + kXSub / 2, &xim, xs * 128 + 64, tb * kTok, &xfull[xst]);
         }
         __syncwarp();
       }
@@ -236,27 +242,28 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ---------------- MMA issuers: warp 8 the sigma plane, warp 9 the tau plane ----------------
     const int e = warp - kIssWarp;
     if (lane == 0) {
-      int p = 0, xq = 0;
-      const int npt = a.wpr / 2;   // step pairs per tile (a tile has 4 steps per x stage)
+      int g = 0;   // running group counter
+      const uint32_t dcol = tmem + kColD + e * 128;
       for (int it = 0; it < my_tiles; ++it) {
         if (it > 0 && !wait_or_abort(dempty, (it - 1) & 1, abort_flag, a.status)) break;
         tc_fence_after();
         bool ok = true;
-        for (int pp = 0; pp < npt && ok; ++pp, ++p) {
-          const int xst = xq % kXS;
-          if ((pp & 1) == 0) ok = wait_or_abort(&xfull[xst], (xq / kXS) & 1, abort_flag, a.status);
-          ok = ok && wait_or_abort(&afull[p % kPairs], (p / kPairs) & 1, abort_flag, a.status);
-          if (!ok) break;
-          tc_fence_after();
-          const uint32_t xaddr = smem_u32(smem + kOffX + xst * kXStage) + (pp & 1) * 64;
-          const uint32_t acol = tmem + kColA + (p % kPairs) * 32 + e * 8;
-          mma_bf16_ts(tmem + kColD + e * 128, acol, smem_desc_sw128(xaddr), pp > 0 ? 1u : 0u);
-          mma_bf16_ts(tmem + kColD + e * 128, acol + 16, smem_desc_sw128(xaddr + 32), 1u);
-          mma_commit(&aempty[p % kPairs]);
-          if (pp & 1) {
-            mma_commit(&xempty[xst]);
-            ++xq;
+        for (int gi = 0; gi < gpt; ++gi, ++g) {
+          const int slot = g % kG;
+          const int xst = (it * nch + (gi >> 1)) % kXS;
+          if (!wait_or_abort(&gfull[slot], (g / kG) & 1, abort_flag, a.status)) {
+            ok = false;
+            break;
           }
+          tc_fence_after();
+          const uint32_t xaddr = smem_u32(smem + kOffX + xst * kXStage + (gi & 1) * kXSub);
+          const uint32_t acol = tmem + kColA + slot * 64 + e * 8;
+#pragma unroll
+          for (int k = 0; k < 4; ++k)   // step k of the group: pair k / 2, step k % 2 of the pair
+            mma_bf16_ts(dcol, acol + (k >> 1) * 32 + (k & 1) * 16, smem_desc_sw128(xaddr + k * 32),
+                        (gi > 0 || k > 0) ? 1u : 0u);
+          mma_commit(&gempty[slot]);
+          if (gi & 1) mma_commit(&xempty[xst]);
         }
         if (!ok) break;
         mma_commit(accf);
@@ -271,9 +278,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int set = warp >> 2, quarter = warp & 3, L = quarter * 32 + lane;
     const uint32_t t_lane = tmem + ((uint32_t)(quarter * 32) << 16);
     const int tl = L >> 4, rl = L & 15;   // 16-row tile (tm * RT + rt) and row within it
-    const int npt = a.wpr / 2;            // step pairs per tile
-    constexpr int kPairsPerStage = kWordsPerStage / 2;
-    float* sred = red + set * (16 * 2 * 128);
+    const bool relay = warp == 0;         // waits for each x stage before arriving on its groups
+    float* sred = red + set * kRedSet;
+    int g = 0;                            // running group counter
     int cq0 = 0;                          // code stages of the earlier tiles
     uint32_t eph = 0;                     // phases of this set's epilogue barrier passed
     // Barrier of the set's 128 threads with a bounded wait (false: the kernel aborts).
@@ -291,40 +298,45 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int it = 0; it < my_tiles; ++it) {
       const int tile = (int)blockIdx.x + it * (int)gridDim.x;
       const int rb = tile % a.row_blocks, tb = tile / a.row_blocks;
-      const int nstages = (npt + kPairsPerStage - 1) / kPairsPerStage;
       bool ok = true;
-      for (int pp = set; pp < npt && ok; pp += 2) {
-        const int p = it * npt + pp;
-        const int g = pp / kPairsPerStage, cq = cq0 + g, st = cq % kCS;
-        ok = __all_sync(0xffffffffu, wait_or_abort(&cfull[st], (cq / kCS) & 1, abort_flag, a.status));
-        if (ok && p >= kPairs)
-          ok = __all_sync(0xffffffffu, wait_or_abort(&aempty[p % kPairs], ((p / kPairs) - 1) & 1,
+      for (int gi = 0; gi < gpt; ++gi, ++g) {
+        const int slot = g % kG;
+        const int cq = cq0 + gi / kGroupsPerCStage, st = cq % kCS;
+        if (gi % kGroupsPerCStage == 0)
+          ok = __all_sync(0xffffffffu, wait_or_abort(&cfull[st], (cq / kCS) & 1, abort_flag, a.status));
+        if (ok && g >= kG)
+          ok = __all_sync(0xffffffffu, wait_or_abort(&gempty[slot], ((g / kG) - 1) & 1,
                                                      abort_flag, a.status));
         if (!ok) break;
-        const int wi = (pp % kPairsPerStage) * 2;   // first word of the pair in the stage
+        const int wi = (gi % kGroupsPerCStage) * 4 + set * 2;   // first word of the pair in the stage
         const uint2 w2 = *reinterpret_cast<const uint2*>(
             smem + kOffCodes + st * kCStage + (tl * kCChunks + (wi >> 3)) * 512 + rl * 32 +
             (wi & 7) * 4);
         uint32_t r[32];
-        uint32_t* rp = r;
-        plane_bf16(prmt(w2.x, 0u, 0x1404u), *reinterpret_cast<uint32_t(*)[8]>(rp));       // sigma, step 2pp
-        plane_bf16(prmt(w2.x, 0u, 0x3424u), *reinterpret_cast<uint32_t(*)[8]>(rp + 8));   // tau
-        plane_bf16(prmt(w2.y, 0u, 0x1404u), *reinterpret_cast<uint32_t(*)[8]>(rp + 16));  // sigma, 2pp+1
-        plane_bf16(prmt(w2.y, 0u, 0x3424u), *reinterpret_cast<uint32_t(*)[8]>(rp + 24));  // tau
-        const bool last_in_stage =
-            pp + 2 >= min((g + 1) * kPairsPerStage, npt);   // this set's last pair of the stage
+        plane_bf16(prmt(w2.x, 0u, 0x1404u), r);        // sigma, first step of the pair
+        plane_bf16(prmt(w2.x, 0u, 0x3424u), r + 8);    // tau
+        plane_bf16(prmt(w2.y, 0u, 0x1404u), r + 16);   // sigma, second step
+        plane_bf16(prmt(w2.y, 0u, 0x3424u), r + 24);   // tau
         __syncwarp();
-        if (lane == 0 && last_in_stage) mbar_arrive(&cempty[st]);
-        tmem_st32(t_lane + kColA + (p % kPairs) * 32, r);
+        if (lane == 0 && (gi % kGroupsPerCStage == kGroupsPerCStage - 1 || gi == gpt - 1))
+          mbar_arrive(&cempty[st]);   // this warp's last read of the code stage
+        tmem_st32(t_lane + kColA + slot * 64 + set * 32, r);
+        if (relay && (gi & 1) == 0) {
+          const int xq = it * nch + (gi >> 1);
+          bool okx = true;
+          if (lane == 0) okx = wait_or_abort(&xfull[xq % kXS], (xq / kXS) & 1, abort_flag, a.status);
+          ok = __shfl_sync(0xffffffffu, okx, 0);
+        }
         tmem_wait_st();
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&afull[p % kPairs]);
+        if (!ok) break;
+        if (lane == 0) mbar_arrive(&gfull[slot]);
       }
-      cq0 += nstages;
+      cq0 += (gpt + kGroupsPerCStage - 1) / kGroupsPerCStage;
       if (!ok) break;
 
-      // ---- epilogue of the tile: set s takes tokens 32 s .. 32 s + 31, in blocks of 16 ----
+      // ---- epilogue: set s takes tokens 32 s .. 32 s + 31 (sub-blocks of 16 tokens) ----
       ok = __all_sync(0xffffffffu, wait_or_abort(accf, it & 1, abort_flag, a.status));
       if (!ok) break;
       tc_fence_after();
@@ -333,6 +345,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int t = tm >> 1, mat = tm & 1;
       const float hr = valid ? 0.5f * __ldg(a.scales + (t * 2 + mat) * 2 + 0) : 0.f;
       const float hi = valid ? 0.5f * __ldg(a.scales + (t * 2 + mat) * 2 + 1) : 0.f;
+#pragma unroll 1
       for (int sb2 = 0; sb2 < 2; ++sb2) {
         const int sb = set * 2 + sb2;
         float pr[16], pi[16], qr[16], qi[16];
@@ -341,11 +354,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_ld16(t_lane + kColD + 128 + sb * 16, qr);
         tmem_ld16(t_lane + kColD + 192 + sb * 16, qi);
         tmem_wait_ld();
-        if (sb2 == 1) {
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(dempty);   // the issuers may start the next tile
-        }
+        float* sr = sred + sb2 * (16 * 2 * 128);
 #pragma unroll
         for (int k = 0; k < 16; ++k) {
           float Pr = pr[k], Pi = pi[k], Qr = qr[k], Qi = qi[k];
@@ -353,25 +362,30 @@ __global__ void __launch_bounds__(kThreads, 1)
             Pi = -Pi;
             Qi = -Qi;
           }
-          sred[(k * 2 + 0) * 128 + L] = valid ? hr * Pr - hi * Pi + hr * Qr + hi * Qi : 0.f;
-          sred[(k * 2 + 1) * 128 + L] = valid ? hr * Pi + hi * Pr + hr * Qi - hi * Qr : 0.f;
+          sr[(k * 2 + 0) * 128 + L] = valid ? hr * Pr - hi * Pi + hr * Qr + hi * Qi : 0.f;
+          sr[(k * 2 + 1) * 128 + L] = valid ? hr * Pi + hi * Pr + hr * Qi - hi * Qr : 0.f;
         }
-        if (!set_sync()) break;
-        // sum over the stage-matrices; item = (token k, part, row r)
-        for (int item = L; item < 16 * 2 * R; item += 128) {
-          const int rr = item % R, kp = item / R;
-          float sum = 0.f;
-#pragma unroll
-          for (int m2 = 0; m2 < TM; ++m2) sum += sred[kp * 128 + m2 * R + rr];
-          const int64_t b = (int64_t)tb * kTok + sb * 16 + (kp >> 1);
-          const int64_t j = (int64_t)rb * R + rr;
-          if (b < a.B && j < a.n) {
-            if ((kp & 1) == 0) a.y[b * a.ldy + j] = sum;
-            else if (a.n + j < a.out_features) a.y[b * a.ldy + a.n + j] = sum;
-          }
-        }
-        if (!set_sync()) break;
       }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(dempty);   // the issuers may start the next tile
+      if (!set_sync()) break;
+      // sum over the stage-matrices; item = (sub-block, token k, part, row r)
+      for (int item = L; item < 2 * 16 * 2 * R; item += 128) {
+        const int sb2 = item / (32 * R), rem = item % (32 * R);
+        const int rr = rem % R, kp = rem / R;
+        const float* sr = sred + sb2 * (16 * 2 * 128) + kp * 128 + rr;
+        float sum = 0.f;
+#pragma unroll
+        for (int m2 = 0; m2 < TM; ++m2) sum += sr[m2 * R];
+        const int64_t b = (int64_t)tb * kTok + (set * 2 + sb2) * 16 + (kp >> 1);
+        const int64_t j = (int64_t)rb * R + rr;
+        if (b < a.B && j < a.n) {
+          if ((kp & 1) == 0) a.y[b * a.ldy + j] = sum;
+          else if (a.n + j < a.out_features) a.y[b * a.ldy + a.n + j] = sum;
+        }
+      }
+      if (!set_sync()) break;
       if (__shfl_sync(0xffffffffu, *abort_flag, 0)) break;
     }
   }
