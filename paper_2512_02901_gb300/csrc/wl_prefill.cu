@@ -23,13 +23,13 @@
 // are stored and x has landed) and one commit (plus one per x stage): the issue cost per MMA is
 // what bounds this kernel once the waits are per MMA.
 //
-// Roles (11 warps): warps 0-7, two sets of four (warp w reaches TMEM lanes 32 (w % 4) ..), decode
+// Roles (15 warps; warp w reaches TMEM lanes 32 (w % 4) ..): warps 0-7, two sets of four, decode
 // the code words into the A ring, set s taking pair s of every group (one 32-column store: sigma,
-// tau of two steps), warp 0 also relaying the x-stage arrival into the group barrier; then they run
-// the epilogue of each tile, set s for tokens 32 s .. 32 s + 31 (all accumulator columns are read
-// out first, so the MMAs of the next tile start before the reduction and the stores). Warps 8 and
-// 9 issue the sigma and the tau MMAs; warp 10 copies the codes (bulk copies of whole 16-row tiles)
-// and x (TMA) in.
+// tau of two steps, left in flight while the next group is decoded), warp 0 also relaying the
+// x-stage arrival into the group barrier; they run on into the next tile without a pause. Warps
+// 8 and 9 issue the sigma and the tau MMAs; warp 10 copies the codes (bulk copies of whole 16-row
+// tiles) and x (TMA) in; warps 11-14 run the epilogue of each tile (every accumulator column is
+// read out first, so the MMAs of the next tile start before the reduction and the stores).
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
@@ -44,9 +44,10 @@ namespace fairy2i {
 
 namespace pfl {
 
-constexpr int kThreads = 11 * 32;
-constexpr int kIssWarp = 8;                       // warps 8, 9: sigma / tau issuers
-constexpr int kCopyWarp = 10;
+constexpr int kIssWarp = 8;                       // warps 0-7 decode; 8, 9: sigma / tau issuers
+constexpr int kCopyWarp = kIssWarp + 2;
+constexpr int kEpiWarp = kCopyWarp + 1;           // 4 epilogue warps
+constexpr int kThreads = (kEpiWarp + 4) * 32;
 constexpr int kTok = 64;                          // tokens per tile
 constexpr int kG = 4;                             // A ring: groups of 64 codes (4 steps)
 constexpr int kColD = 0;                          // sigma accumulator: columns 0-127, tau 128-255
@@ -59,7 +60,7 @@ constexpr int kCChunks = 2;                       // 128-code chunks per code st
 constexpr int kCS = 3;                            // code stages
 constexpr int kCStage = kCChunks * 8 * 512;       // <= 8 tiles x kCChunks x 512 B
 constexpr int kGroupsPerCStage = 2 * kCChunks;
-constexpr int kRedSet = 2 * 16 * 2 * 128;         // floats: [sub-block][16 tokens][2][128 lanes]
+constexpr int kRed = 4 * 16 * 2 * 128;            // floats: [sub-block][16 tokens][2][128 lanes]
 constexpr uint64_t kWaitNs = 1000000000ull;
 // kind::f16, bf16 A and B (format 1), f32 D, K-major, N = 128, M = 128.
 constexpr uint32_t kIdesc =
@@ -68,8 +69,8 @@ constexpr uint32_t kIdesc =
 constexpr int kOffX = 0;                                        // 1024-aligned (swizzle 128 B)
 constexpr int kOffCodes = kOffX + kXS * kXStage;                // 128 KB
 constexpr int kOffRed = kOffCodes + kCS * kCStage;              // + 24 KB
-constexpr int kOffBar = kOffRed + 2 * kRedSet * 4;              // + 64 KB
-constexpr int kNumBars = 2 * kXS + 2 * kCS + 2 * kG + 6;
+constexpr int kOffBar = kOffRed + kRed * 4;                     // + 64 KB
+constexpr int kNumBars = 2 * kXS + 2 * kCS + 2 * kG + 5;
 constexpr int kOffMisc = kOffBar + kNumBars * 8;
 constexpr int kSmemBytes = kOffMisc + 64 + 1024;
 static_assert(kSmemBytes > 116 * 1024, "one CTA per SM: it owns all TMEM columns");
@@ -137,12 +138,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* xempty = xfull + kXS;           // x stage consumed          (2 issuer commits)
   uint64_t* cfull = xempty + kXS;           // code stage landed         (tx)
   uint64_t* cempty = cfull + kCS;           // code stage read           (8 decoder warps)
-  uint64_t* gfull = cempty + kCS;           // group's A stored, x in    (8 decoder warps)
+  uint64_t* gfull = cempty + kCS;           // group's A stored, x in    (4 warps x 2 pairs)
   uint64_t* gempty = gfull + kG;            // group's A consumed        (2 issuer commits)
   uint64_t* accf = gempty + kG;             // tile accumulators final   (2 issuer commits)
-  uint64_t* dempty = accf + 1;              // accumulators read out     (8 decoder warps)
+  uint64_t* dempty = accf + 1;              // accumulators read out     (4 epilogue warps)
   uint64_t* fin = dempty + 1;               // [2] issued MMAs complete (end of kernel)
-  uint64_t* ebar = fin + 2;                 // [2] epilogue barrier of a decoder set (128 threads)
+  uint64_t* ebar = fin + 2;                 // epilogue warps' barrier (128 threads)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + kOffMisc);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kOffMisc + 8);
   float* red = reinterpret_cast<float*>(smem + kOffRed);
@@ -167,11 +168,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&gempty[i], 2);
     }
     mbar_init(accf, 2);
-    mbar_init(dempty, 8);
+    mbar_init(dempty, 4);
     mbar_init(&fin[0], 1);
     mbar_init(&fin[1], 1);
-    mbar_init(&ebar[0], 128);
-    mbar_init(&ebar[1], 128);
+    mbar_init(ebar, 128);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -273,40 +273,30 @@ __global__ void __launch_bounds__(kThreads, 1)
       (void)mbar_wait_timed(&fin[e], 0, kWaitNs);
     }
     __syncwarp();
-  } else {
-    // ---------------- warps 0-7: decode + epilogue ----------------
+  } else if (warp < kIssWarp) {
+    // ---------------- warps 0-7: decode ----------------
     const int set = warp >> 2, quarter = warp & 3, L = quarter * 32 + lane;
     const uint32_t t_lane = tmem + ((uint32_t)(quarter * 32) << 16);
     const int tl = L >> 4, rl = L & 15;   // 16-row tile (tm * RT + rt) and row within it
     const bool relay = warp == 0;         // waits for each x stage before arriving on its groups
-    float* sred = red + set * kRedSet;
     int g = 0;                            // running group counter
     int cq0 = 0;                          // code stages of the earlier tiles
-    uint32_t eph = 0;                     // phases of this set's epilogue barrier passed
-    // Barrier of the set's 128 threads with a bounded wait (false: the kernel aborts).
-    auto set_sync = [&]() -> bool {
-      mbar_arrive(&ebar[set]);
-      const bool ok = mbar_wait_timed(&ebar[set], eph & 1, kWaitNs);
-      ++eph;
-      if (!__all_sync(0xffffffffu, ok)) {
-        *abort_flag = 1;
-        if (lane == 0) latch_status(a.status, kStatusTimeout);
-        return false;
-      }
-      return true;
-    };
     for (int it = 0; it < my_tiles; ++it) {
-      const int tile = (int)blockIdx.x + it * (int)gridDim.x;
-      const int rb = tile % a.row_blocks, tb = tile / a.row_blocks;
       bool ok = true;
+      // Software pipeline of one group: the A store of group g is in flight while group g + 1 is
+      // decoded; its barrier arrival follows the store wait at the next iteration.
+      int pend = -1;                      // slot of the group stored but not yet announced
       for (int gi = 0; gi < gpt; ++gi, ++g) {
         const int slot = g % kG;
         const int cq = cq0 + gi / kGroupsPerCStage, st = cq % kCS;
         if (gi % kGroupsPerCStage == 0)
           ok = __all_sync(0xffffffffu, wait_or_abort(&cfull[st], (cq / kCS) & 1, abort_flag, a.status));
-        if (ok && g >= kG)
-          ok = __all_sync(0xffffffffu, wait_or_abort(&gempty[slot], ((g / kG) - 1) & 1,
-                                                     abort_flag, a.status));
+        if (ok && relay && (gi & 1) == 0) {   // x of this group landed (announced with the group)
+          const int xq = it * nch + (gi >> 1);
+          bool okx = true;
+          if (lane == 0) okx = wait_or_abort(&xfull[xq % kXS], (xq / kXS) & 1, abort_flag, a.status);
+          ok = __shfl_sync(0xffffffffu, okx, 0);
+        }
         if (!ok) break;
         const int wi = (gi % kGroupsPerCStage) * 4 + set * 2;   // first word of the pair in the stage
         const uint2 w2 = *reinterpret_cast<const uint2*>(
@@ -320,41 +310,65 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
         if (lane == 0 && (gi % kGroupsPerCStage == kGroupsPerCStage - 1 || gi == gpt - 1))
           mbar_arrive(&cempty[st]);   // this warp's last read of the code stage
-        tmem_st32(t_lane + kColA + slot * 64 + set * 32, r);
-        if (relay && (gi & 1) == 0) {
-          const int xq = it * nch + (gi >> 1);
-          bool okx = true;
-          if (lane == 0) okx = wait_or_abort(&xfull[xq % kXS], (xq / kXS) & 1, abort_flag, a.status);
-          ok = __shfl_sync(0xffffffffu, okx, 0);
+        if (pend >= 0) {
+          tmem_wait_st();
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&gfull[pend]);
+          pend = -1;
         }
+        if (g >= kG)
+          ok = __all_sync(0xffffffffu, wait_or_abort(&gempty[slot], ((g / kG) - 1) & 1,
+                                                     abort_flag, a.status));
+        if (!ok) break;
+        tmem_st32(t_lane + kColA + slot * 64 + set * 32, r);
+        pend = slot;
+      }
+      if (ok && pend >= 0) {
         tmem_wait_st();
         tc_fence_before();
         __syncwarp();
-        if (!ok) break;
-        if (lane == 0) mbar_arrive(&gfull[slot]);
+        if (lane == 0) mbar_arrive(&gfull[pend]);
       }
       cq0 += (gpt + kGroupsPerCStage - 1) / kGroupsPerCStage;
       if (!ok) break;
-
-      // ---- epilogue: set s takes tokens 32 s .. 32 s + 31 (sub-blocks of 16 tokens) ----
-      ok = __all_sync(0xffffffffu, wait_or_abort(accf, it & 1, abort_flag, a.status));
-      if (!ok) break;
+    }
+  } else {
+    // ---------------- warps kEpiWarp .. kEpiWarp + 3: epilogue of each tile ----------------
+    const int quarter = warp & 3, L = quarter * 32 + lane;
+    const uint32_t t_lane = tmem + ((uint32_t)(quarter * 32) << 16);
+    const int tm = L / R;
+    const bool valid = L < TM * R;
+    const int t = tm >> 1, mat = tm & 1;
+    const float hr = valid ? 0.5f * __ldg(a.scales + (t * 2 + mat) * 2 + 0) : 0.f;
+    const float hi = valid ? 0.5f * __ldg(a.scales + (t * 2 + mat) * 2 + 1) : 0.f;
+    uint32_t eph = 0;                     // phases of the epilogue barrier passed
+    // Barrier of the 128 epilogue threads with a bounded wait (false: the kernel aborts).
+    auto epi_sync = [&]() -> bool {
+      mbar_arrive(ebar);
+      const bool ok = mbar_wait_timed(ebar, eph & 1, kWaitNs);
+      ++eph;
+      if (!__all_sync(0xffffffffu, ok)) {
+        *abort_flag = 1;
+        if (lane == 0) latch_status(a.status, kStatusTimeout);
+        return false;
+      }
+      return true;
+    };
+    for (int it = 0; it < my_tiles; ++it) {
+      const int tile = (int)blockIdx.x + it * (int)gridDim.x;
+      const int rb = tile % a.row_blocks, tb = tile / a.row_blocks;
+      if (!__all_sync(0xffffffffu, wait_or_abort(accf, it & 1, abort_flag, a.status))) break;
       tc_fence_after();
-      const int tm = L / R;
-      const bool valid = L < TM * R;
-      const int t = tm >> 1, mat = tm & 1;
-      const float hr = valid ? 0.5f * __ldg(a.scales + (t * 2 + mat) * 2 + 0) : 0.f;
-      const float hi = valid ? 0.5f * __ldg(a.scales + (t * 2 + mat) * 2 + 1) : 0.f;
 #pragma unroll 1
-      for (int sb2 = 0; sb2 < 2; ++sb2) {
-        const int sb = set * 2 + sb2;
+      for (int sb = 0; sb < 4; ++sb) {   // 16 tokens per sub-block
         float pr[16], pi[16], qr[16], qi[16];
         tmem_ld16(t_lane + kColD + sb * 16, pr);
         tmem_ld16(t_lane + kColD + 64 + sb * 16, pi);
         tmem_ld16(t_lane + kColD + 128 + sb * 16, qr);
         tmem_ld16(t_lane + kColD + 192 + sb * 16, qi);
         tmem_wait_ld();
-        float* sr = sred + sb2 * (16 * 2 * 128);
+        float* sr = red + sb * (16 * 2 * 128);
 #pragma unroll
         for (int k = 0; k < 16; ++k) {
           float Pr = pr[k], Pi = pi[k], Qr = qr[k], Qi = qi[k];
@@ -369,23 +383,23 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(dempty);   // the issuers may start the next tile
-      if (!set_sync()) break;
+      if (!epi_sync()) break;
       // sum over the stage-matrices; item = (sub-block, token k, part, row r)
-      for (int item = L; item < 2 * 16 * 2 * R; item += 128) {
-        const int sb2 = item / (32 * R), rem = item % (32 * R);
+      for (int item = L; item < 4 * 16 * 2 * R; item += 128) {
+        const int sb = item / (32 * R), rem = item % (32 * R);
         const int rr = rem % R, kp = rem / R;
-        const float* sr = sred + sb2 * (16 * 2 * 128) + kp * 128 + rr;
+        const float* sr = red + sb * (16 * 2 * 128) + kp * 128 + rr;
         float sum = 0.f;
 #pragma unroll
         for (int m2 = 0; m2 < TM; ++m2) sum += sr[m2 * R];
-        const int64_t b = (int64_t)tb * kTok + (set * 2 + sb2) * 16 + (kp >> 1);
+        const int64_t b = (int64_t)tb * kTok + sb * 16 + (kp >> 1);
         const int64_t j = (int64_t)rb * R + rr;
         if (b < a.B && j < a.n) {
           if ((kp & 1) == 0) a.y[b * a.ldy + j] = sum;
           else if (a.n + j < a.out_features) a.y[b * a.ldy + a.n + j] = sum;
         }
       }
-      if (!set_sync()) break;
+      if (!epi_sync()) break;
       if (__shfl_sync(0xffffffffu, *abort_flag, 0)) break;
     }
   }
