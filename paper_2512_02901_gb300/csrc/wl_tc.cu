@@ -157,19 +157,6 @@ __device__ __forceinline__ void pow2_scale(float mx, float& S, float& invS) {
   }
 }
 
-// e4m3 limbs of eight bf16 values scaled by S: hi = e4m3(v S) rounded to nearest, lo =
-// e4m3(64 (v S - hi)); returned as byte pairs (values 2i, 2i+1 in register i).
-__device__ __forceinline__ void limbs8(const uint4& xv, float S, uint32_t (&hw)[4], uint32_t (&lw)[4]) {
-  const uint32_t e[4] = {xv.x, xv.y, xv.z, xv.w};
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const float v0 = bf_lo(e[i]) * S, v1 = bf_hi(e[i]) * S;
-    hw[i] = e4m3x2(v0, v1);
-    const float2 hf = e4m3x2_to_float2(hw[i]);
-    lw[i] = e4m3x2(64.f * (v0 - hf.x), 64.f * (v1 - hf.y));
-  }
-}
-
 // Row n of a word's B tile, K bytes 16 hh .. 16 hh + 15 (core matrices of 8 rows x 16 bytes,
 // K-adjacent at +128, 8-row groups at +256).
 __device__ __forceinline__ void store_brow(unsigned char* tile, int n, int hh, uint4 v) {
@@ -280,21 +267,19 @@ __global__ void __launch_bounds__(kThreads, 1) wl_tc_decode_kernel(const Args a)
     // ------------- sets: decode a unit into a slot, then two warps issue its MMAs -------------
     const int set = warp >> 2, quarter = warp & 3;
     const int L = quarter * 32 + lane;
-    const bool issuer = quarter < 2 && lane == 0;
     const uint32_t codes_addr =
         smem_u32(smem + kOffCodes) + (uint32_t)((L >> 4) * kGU * 512 + (L & 15) * 32);
     const uint32_t t_lane = tmem + ((uint32_t)(quarter * 32) << 16) + kColA;
-    const uint32_t d_tmem = tmem + (set * 2 + quarter) * 16;   // accumulator of an issuer
-    const uint32_t b_base = smem_u32(smem + kOffB);
-    bool b_ok = false, issued = false;
     int j = 0;
+    // Software pipeline: the A stores of unit j are announced once the first half of unit j + 1
+    // is decoded (the store wait then finds them done).
+    int pend = -1;          // slot written but not yet announced
+    bool ok = true;
     for (int u = set; u < units; u += kSets, ++j) {
       const int sl = j % kSlots, g = u / kGU, ui = u - g * kGU, st = g % kSG;
       const int si = set * kSlots + sl;
-      bool ok = wait_or_abort(&cfull[st], (g / kSG) & 1, abort_flag, a.status);
-      if (j >= kSlots)   // the slot's previous unit has been consumed
-        ok = ok && wait_or_abort(&sfree[si], ((j / kSlots) - 1) & 1, abort_flag, a.status);
-      if (!__all_sync(0xffffffffu, ok)) break;
+      ok = __all_sync(0xffffffffu, wait_or_abort(&cfull[st], (g / kSG) & 1, abort_flag, a.status));
+      if (!ok) break;
       const uint32_t src = codes_addr + st * kGU * kUnitBytes + ui * 512;
       const uint4 q0 = lds128(src), q1 = lds128(src + 16);
       const uint32_t a_col = t_lane + si * 64;
@@ -303,43 +288,32 @@ __global__ void __launch_bounds__(kThreads, 1) wl_tc_decode_kernel(const Args a)
       decode_word(q0.y, r + 8);
       decode_word(q0.z, r + 16);
       decode_word(q0.w, r + 24);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&cempty[st]);
+      if (pend >= 0) {
+        tmem_wait_st();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sfull[pend]);
+        pend = -1;
+      }
+      if (j >= kSlots)   // the slot's previous unit has been consumed
+        ok = __all_sync(0xffffffffu, wait_or_abort(&sfree[si], ((j / kSlots) - 1) & 1, abort_flag,
+                                                   a.status));
+      if (!ok) break;
       tmem_st32(a_col, r);
       decode_word(q1.x, r);
       decode_word(q1.y, r + 8);
       decode_word(q1.z, r + 16);
       decode_word(q1.w, r + 24);
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&cempty[st]);
       tmem_st32(a_col + 32, r);
+      pend = si;
+    }
+    if (ok && pend >= 0) {
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&sfull[si]);
-      if (issuer) {
-        // words 4 quarter .. 4 quarter + 3 of unit u, once the set's four warps have written it
-        bool go = wait_or_abort(&sfull[si], (j / kSlots) & 1, abort_flag, a.status);
-        if (go && !b_ok) go = b_ok = wait_or_abort(bready, 0, abort_flag, a.status);
-        if (go) {
-          tc_fence_after();
-          const uint32_t a_slot = tmem + kColA + si * 64;
-#pragma unroll
-          for (int w4 = 0; w4 < 4; ++w4) {
-            const int wd = quarter * 4 + w4;
-            mma_e4m3_ts(d_tmem, a_slot + wd * 8,
-                        smem_desc(b_base + u * kUnitB + wd * kWordB, 128, 256), kIdesc,
-                        (j > 0 || w4 > 0) ? 1u : 0u);
-          }
-          issued = true;
-          mma_commit(&sfree[si]);
-          if (u + kSets >= units) mma_commit(&sdone[set]);
-        }
-      }
-      __syncwarp();
-    }
-    // Abort path: MMAs this thread issued must finish before TMEM is released.
-    if (issuer && issued && *abort_flag) {
-      mma_commit(&fin[set * 2 + quarter]);
-      (void)mbar_wait_timed(&fin[set * 2 + quarter], 0, kWaitNs);
+      if (lane == 0) mbar_arrive(&sfull[pend]);
     }
 
     // ---- epilogue: each warp sums its set's two accumulators for its 32 lanes ----
@@ -451,6 +425,14 @@ __global__ void __launch_bounds__(kThreads, 1) wl_tc_decode_kernel(const Args a)
     }
   } else if (warp == kCopyWarp) {
     // ---------------- copies: x slice (after the programmatic wait), then the codes ----------
+    if (a.x_bulk && lane < 2 * NB && lane / 2 < a.B) {
+      // Warm L2 with this CTA's x slice; the copy below (after the wait) reads the final values.
+      const int b = lane >> 1, p = lane & 1;
+      const int64_t lim = p ? a.in_features - a.m : a.m;
+      const int64_t k0 = (int64_t)c0 * 128, k1 = min((int64_t)(c0 + units) * 128, lim);
+      if (k1 > k0)
+        prefetch_l2_bulk(a.x + (int64_t)b * a.ldx + (int64_t)p * a.m + k0, (uint32_t)((k1 - k0) * 2));
+    }
     pdl_wait_primary();   // x may be written by the previous kernel
     if (a.x_bulk) {
       // per (token, part): complex indices [c0 128, min((c0 + units) 128, lim)) of the row
@@ -539,47 +521,93 @@ __global__ void __launch_bounds__(kThreads, 1) wl_tc_decode_kernel(const Args a)
     // B tiles: task (unit, token, word, half, row): one 16-byte row half per lane, the eight lanes
     // of a shared-memory phase writing the eight rows of one core matrix (no bank conflicts).
     // Row n = ((b 2 + limb) 2 + slot) 2 + p holds the limb bytes of codes 2j', 2j'+1 in the sigma
-    // half (bytes 0-1) or the tau half (bytes 2-3) of register j'.
-    for (int q = xt; q < NB * units * 128; q += kXThreads) {
+    // half (bytes 0-1) or the tau half (bytes 2-3) of register j'. The eight lanes of a row group
+    // convert the 16 values of the group once (lane nl: values 2 (nl & 3), + 1 of part nl >> 2)
+    // and exchange the limb pairs by shuffles.
+    for (int q = xt; q < NB * units * 128; q += kXThreads) {   // warp-uniform: multiples of 32
       const int nl = q & 7, hh = (q >> 3) & 1, wd = (q >> 4) & 7, rest = q >> 7;
       const int b = rest % NB, u = rest / NB;
       const int limb = nl >> 2, slot = (nl >> 1) & 1, p = nl & 1;
-      const uint4 xv = *reinterpret_cast<const uint4*>(
-          xs + (b * 2 + p) * kMaxUnits * 128 + u * 128 + wd * 16 + hh * 8);
-      uint32_t hw[4], lw[4];
-      limbs8(xv, S[b], hw, lw);
+      const uint32_t e2 = *reinterpret_cast<const uint32_t*>(
+          xs + (b * 2 + (nl >> 2)) * kMaxUnits * 128 + u * 128 + wd * 16 + hh * 8 + 2 * (nl & 3));
+      const float v0 = bf_lo(e2) * S[b], v1 = bf_hi(e2) * S[b];
+      const uint32_t hp = e4m3x2(v0, v1) & 0xffffu;
+      const float2 hf = e4m3x2_to_float2(hp);
+      const uint32_t lp = e4m3x2(64.f * (v0 - hf.x), 64.f * (v1 - hf.y)) & 0xffffu;
+      const uint32_t both = hp | (lp << 16);
       uint32_t w[4];
 #pragma unroll
-      for (int i = 0; i < 4; ++i) w[i] = (limb ? lw[i] : hw[i]) << (slot ? 16 : 0);
+      for (int i = 0; i < 4; ++i) {
+        const uint32_t v = __shfl_sync(0xffffffffu, both, (lane & ~7) | (p * 4 + i));
+        w[i] = (limb ? (v >> 16) : (v & 0xffffu)) << (slot ? 16 : 0);
+      }
       store_brow(smem + kOffB + u * kUnitB + wd * kWordB, b * 8 + nl, hh,
                  make_uint4(w[0], w[1], w[2], w[3]));
     }
     fence_proxy_async_smem();
     named_bar_sync(3, kXThreads);
     if (xt == 0) mbar_arrive(bready);
-    // C term (needed by the epilogue only): task (token, chunk, part, 8 values)
-    for (int q = xt; q < NB * units * 32; q += kXThreads) {   // warp-uniform: multiples of 32
-      const int v = q & 15, p = (q >> 4) & 1, lc = (q >> 5) % units, b = (q >> 5) / units;
-      const uint4 u4 =
-          *reinterpret_cast<const uint4*>(xs + (b * 2 + p) * kMaxUnits * 128 + lc * 128 + v * 8);
-      const uint32_t e[4] = {u4.x, u4.y, u4.z, u4.w};
-      // 1 + alpha of codes 8h .. 8h + 7 of a word (h = v & 1): 5,5,3,3,5,5,3,3 or 1,1,0,0,..
-      const float p0 = bf_lo(e[0]) + bf_hi(e[0]), p1 = bf_lo(e[1]) + bf_hi(e[1]);
-      const float p2 = bf_lo(e[2]) + bf_hi(e[2]), p3 = bf_lo(e[3]) + bf_hi(e[3]);
-      float cs = (v & 1) ? (p0 + p2) : (5.f * (p0 + p2) + 3.f * (p1 + p3));
+    const int xw = warp - kXWarp0;
+    if (xw < 2 * kSets) {
+      // ------ MMA issuers: lane 0 of x-warp 2 d + e issues words 4 e .. 4 e + 3 of every unit of
+      // set d (its own accumulator), once the set's four warps have written the unit ------
+      const int set = xw >> 1, e = xw & 1;
+      if (lane == 0) {
+        const uint32_t d_tmem = tmem + (set * 2 + e) * 16;
+        const uint32_t b_base = smem_u32(smem + kOffB);
+        bool issued = false;
+        int j = 0;
+        for (int u = set; u < units; u += kSets, ++j) {
+          const int si = set * kSlots + j % kSlots;
+          if (!wait_or_abort(&sfull[si], (j / kSlots) & 1, abort_flag, a.status)) break;
+          tc_fence_after();
+          const uint32_t a_slot = tmem + kColA + si * 64;
 #pragma unroll
-      for (int h = 8; h >= 1; h >>= 1) cs += __shfl_xor_sync(0xffffffffu, cs, h);
-      if (v == 0) Cch[lc * 4 + b * 2 + p] = cs;
-    }
-    named_bar_sync(3, kXThreads);
-    if (xt < 2 * NB) {
-      float cs = 0.f;
+          for (int w4 = 0; w4 < 4; ++w4) {
+            const int wd = e * 4 + w4;
+            mma_e4m3_ts(d_tmem, a_slot + wd * 8,
+                        smem_desc(b_base + u * kUnitB + wd * kWordB, 128, 256), kIdesc,
+                        (j > 0 || w4 > 0) ? 1u : 0u);
+          }
+          issued = true;
+          mma_commit(&sfree[si]);
+          if (u + kSets >= units) mma_commit(&sdone[set]);
+        }
+        // Abort path: MMAs this thread issued must finish before TMEM is released.
+        if (issued && *abort_flag) {
+          mma_commit(&fin[set * 2 + e]);
+          (void)mbar_wait_timed(&fin[set * 2 + e], 0, kWaitNs);
+        }
+      }
+      __syncwarp();
+    } else {
+      // ------ the other x-warps: C term (needed by the epilogue only) ------
+      constexpr int kCThreads = kXThreads - 2 * kSets * 32;
+      const int ct = xt - 2 * kSets * 32;   // 0 .. kCThreads-1
+      // task (token, chunk, part, 8 values)
+      for (int q = ct; q < NB * units * 32; q += kCThreads) {   // warp-uniform: multiples of 32
+        const int v = q & 15, p = (q >> 4) & 1, lc = (q >> 5) % units, b = (q >> 5) / units;
+        const uint4 u4 =
+            *reinterpret_cast<const uint4*>(xs + (b * 2 + p) * kMaxUnits * 128 + lc * 128 + v * 8);
+        const uint32_t e[4] = {u4.x, u4.y, u4.z, u4.w};
+        // 1 + alpha of codes 8h .. 8h + 7 of a word (h = v & 1): 5,5,3,3,5,5,3,3 or 1,1,0,0,..
+        const float p0 = bf_lo(e[0]) + bf_hi(e[0]), p1 = bf_lo(e[1]) + bf_hi(e[1]);
+        const float p2 = bf_lo(e[2]) + bf_hi(e[2]), p3 = bf_lo(e[3]) + bf_hi(e[3]);
+        float cs = (v & 1) ? (p0 + p2) : (5.f * (p0 + p2) + 3.f * (p1 + p3));
+#pragma unroll
+        for (int h = 8; h >= 1; h >>= 1) cs += __shfl_xor_sync(0xffffffffu, cs, h);
+        if (v == 0) Cch[lc * 4 + b * 2 + p] = cs;
+      }
+      named_bar_sync(4, kCThreads);
+      if (ct < 2 * NB) {
+        float cs = 0.f;
 #pragma unroll 1
-      for (int lc = 0; lc < units; ++lc) cs += Cch[lc * 4 + xt];
-      misc->cseg[xt] = cs;
+        for (int lc = 0; lc < units; ++lc) cs += Cch[lc * 4 + ct];
+        misc->cseg[ct] = cs;
+      }
+      named_bar_sync(4, kCThreads);
+      if (ct == 0) mbar_arrive(cready);
     }
-    named_bar_sync(3, kXThreads);
-    if (xt == 0) mbar_arrive(cready);
   }
 
   // Every thread pairs its cluster arrive (set 0 waited in the epilogue). Rank 0 leaves only after
