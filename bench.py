@@ -51,6 +51,13 @@ def peaks():
         return 6800.0, 1900.0, "fallback"
 
 
+# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) from ncu captures of the current
+# kernels (profiles/wl_decode_fp8_llama2_7b_stack_b1.md, profiles/wl_prefill_llama2_7b_2048tok.md):
+# one decoder layer's seven decode launches (every layer has the same shapes), and one T = 2
+# prefill launch of the 4096 -> 11008 layer on 2048 tokens.
+DECODE_DRAM_BYTES_PER_LAYER = 4 * 4.231e6 + 2 * 11.309e6 + 11.323e6
+PREFILL_T2_UP_DRAM_BYTES = 28.087e6 + 38.276e6
+
 PREFILL_TOKENS = 2048
 PREFILL_LAYERS = (("up", 11008, 4096, 0), ("down", 4096, 11008, 1))   # (name, out, in, seed idx)
 
@@ -279,7 +286,8 @@ def run_ours(args, world, rank, local):
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": launches_per_step * args.steps,
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm,
-                     "unit": "GB/s", "frac": round(achieved / hbm, 4), "traffic": None,
+                     "unit": "GB/s", "frac": round(achieved / hbm, 4),
+                     "traffic": int(DECODE_DRAM_BYTES_PER_LAYER * args.layers),
                      "peak_kind": f"{peak_kind} hbm_gbs (burst copy)",
                      "kernel": "wl_matmul decode (all launches of the step)"},
         "clocks": clk,
@@ -340,7 +348,8 @@ def run_prefill(F, dev, steps: int, warmup: int):
                              "tensor_frac": round(mma / bf16, 4)})
             if name == "up" and T == T_STAGES:
                 roof = {"bound": "tensor", "achieved": round(mma, 1), "peak": bf16,
-                        "unit": "TFLOP/s", "frac": round(mma / bf16, 4), "traffic": None,
+                        "unit": "TFLOP/s", "frac": round(mma / bf16, 4),
+                        "traffic": int(PREFILL_T2_UP_DRAM_BYTES),
                         "peak_kind": f"{peak_kind} bf16_tflops (burst)",
                         "kernel": f"wl_prefill_kernel<{T}> (up {cols}->{rows}, "
                                   f"{PREFILL_TOKENS} tokens)"}

@@ -174,6 +174,16 @@ fairy2i_status fairy2i_wl_matmul_path(const void* x, fairy2i_dtype xdt, int64_t 
  * ------------------------------------------------------------------------------------------ */
 fairy2i_status fairy2i_get_status(void* stream);
 
+/* ------------------------------------------------------------------------------------------
+ * Self-test of the device-side failure detection. Enqueues on `stream` one small kernel that
+ * runs the bounded barrier wait of the matmul kernels' pipelines on a barrier that nothing
+ * completes. After about limit_us microseconds the wait gives up, latches FAIRY2I_ERR_TIMEOUT
+ * in the status word (read and cleared by fairy2i_get_status) and the kernel returns normally,
+ * so the CUDA context stays usable. limit_us must be in 1 .. 100000
+ * (FAIRY2I_ERR_INVALID_ARG otherwise, nothing enqueued); FAIRY2I_ERR_CUDA if the launch fails.
+ * ------------------------------------------------------------------------------------------ */
+fairy2i_status fairy2i_selftest_wait_timeout(uint32_t limit_us, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -34,6 +34,7 @@ SIGNATURES = {
                                 _int, _vp], _int),
     "fairy2i_get_status": ([_vp], _int),
     "fairy2i_quantize_noalloc": ([_vp, _vp, _i64, _i64, _i64, _int, _vp, _vp, _vp], _int),
+    "fairy2i_selftest_wait_timeout": ([_c.c_uint32, _vp], _int),
 }
 
 
@@ -144,6 +145,13 @@ def wl_matmul(x: torch.Tensor, codes: torch.Tensor, scales: torch.Tensor, out_fe
                                          _ptr(scales), out_features, T, _ptr(y), y.stride(0),
                                          path, _stream(stream)))
     return y
+
+
+def selftest_wait_timeout(limit_us: int, stream=None):
+    """Runs the device-side bounded wait on a barrier nothing completes (gives up after about
+    limit_us microseconds and latches the timeout status; read it with get_status)."""
+    _check("fairy2i_selftest_wait_timeout",
+           load().fairy2i_selftest_wait_timeout(limit_us, _stream(stream)))
 
 
 def get_status(stream=None) -> int:

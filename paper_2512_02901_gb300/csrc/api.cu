@@ -29,6 +29,7 @@ fairy2i_status launch_wl_prefill(const void* x, fairy2i_dtype xdt, int64_t B, in
                                  int64_t ldx, const uint32_t* codes, const float* scales,
                                  int64_t n, int64_t m, int64_t out_features, int64_t wpr, int T,
                                  float* y, int64_t ldy, cudaStream_t stream, bool* handled);
+fairy2i_status launch_selftest_wait(uint32_t limit_us, cudaStream_t stream);
 
 // Status word: one __device__ word per device that has loaded the module; its address is
 // looked up once per device with that device current.
@@ -150,6 +151,11 @@ fairy2i_status fairy2i_wl_matmul(const void* x, fairy2i_dtype xdt, int64_t B, in
                                  void* stream) {
   return fairy2i_wl_matmul_path(x, xdt, B, in_features, ldx, codes, scales, out_features, T, y,
                                 ldy, 0, stream);
+}
+
+fairy2i_status fairy2i_selftest_wait_timeout(uint32_t limit_us, void* stream) {
+  if (limit_us < 1 || limit_us > 100000) return FAIRY2I_ERR_INVALID_ARG;
+  return launch_selftest_wait(limit_us, static_cast<cudaStream_t>(stream));
 }
 
 fairy2i_status fairy2i_get_status(void* stream) {

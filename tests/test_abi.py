@@ -93,3 +93,9 @@ def test_wl_matmul_validation(lib):
     assert call(xdt=7) == 4
     assert call(ldx=15) == 2 and call(ldy=15) == 2
     assert call(x=ODD) == 3 and call(codes=ODD) == 3
+
+
+def test_selftest_wait_timeout_validation(lib):
+    """Out-of-range limits are refused before anything is enqueued."""
+    assert lib.fairy2i_selftest_wait_timeout(0, None) == 1
+    assert lib.fairy2i_selftest_wait_timeout(100001, None) == 1

@@ -419,3 +419,19 @@ def test_wl_tcgen05_prefill_rejects_outside_its_domain(F):
                     upload_codes(O.pack_codes(codes5)), torch.from_numpy(scales5).to(DEV),
                     2 * n, path=3)
     assert e.value.code == 1
+
+
+# ------------------------------------------------------------------------------ failure detection
+def test_bounded_wait_latches_timeout_and_context_survives(F):
+    """A bounded wait on a barrier that nothing completes gives up after its limit, latches
+    FAIRY2I_ERR_TIMEOUT, is cleared by reading it, and the context keeps working."""
+    assert F.get_status() == 0
+    F.selftest_wait_timeout(2000)                     # 2 ms
+    assert F.get_status() == 7                        # FAIRY2I_ERR_TIMEOUT
+    assert F.get_status() == 0                        # read and cleared
+    n, m, T, B = 24, 40, 2, 3
+    codes, scales = _random_quantized(n, m, T, seed=31)
+    x = synth.random_matrix(B, 2 * m, seed=32)
+    yg = _run_wl(F, x, codes, scales, 2 * n)
+    xo = x.numpy()
+    assert_wl_close(yg, O.wl_matmul(xo, codes, scales, 2 * n), xo, scales)
