@@ -3,7 +3,8 @@
 Workload (default): 32 decoder layers x {q, k, v, o, gate, up, down} (hidden 4096, intermediate
 11008), every weight Student-t(df=4, std 0.02), converted and quantized with T=2 stages; one
 step = one decode token (batch 1, bf16 activations with 1% outlier channels) through all 224
-quantized linears. Metric: decode GB/s = algorithmic bytes (packed codes + scales + x + y of
+quantized linears, as a decoder layer feeds them: q, k, v on one input (one grouped call), o,
+gate and up on one input (one grouped call), down; 4 calls per layer (--ungrouped: 7). Metric: decode GB/s = algorithmic bytes (packed codes + scales + x + y of
 every linear) per second, against the HBM copy peak. The 1.62 GB of codes per step exceed the
 L2 many times over, so no L2 flush is needed between steps.
 
@@ -158,25 +159,53 @@ def max_over_ranks(v: float, world: int) -> float:
 
 
 # --------------------------------------------------------------------------------------------
-def build_stack(F, layers: int, B: int, dev):
-    """Converts + quantizes every linear of the stack on the GPU; returns per-linear state."""
-    stack = []
-    for (L, pi, name, rows, cols) in layer_shapes(layers):
-        seed = synth.weight_seed("stack", L, pi)
-        R = synth.student_t_weight(rows, cols, seed, device=dev)
-        U, W = F.convert(R)
-        del R
-        codes, scales = F.quantize(U, W, T_STAGES)
-        del U, W
-        x = synth.outlier_activations(B, cols, synth.activation_seed(seed, B), device=dev)
-        y = torch.empty((B, rows), dtype=torch.float32, device=dev)
-        stack.append(dict(L=L, name=name, rows=rows, cols=cols, codes=codes, scales=scales, x=x,
-                          y=y))
+GROUPS = (("q", "k", "v"), ("o",), ("gate", "up"), ("down",))   # linears sharing an input
+
+
+def build_stack(F, layers: int, B: int, dev, grouped: bool = True):
+    """Converts + quantizes every linear of the stack on the GPU; returns the calls of a step:
+    per call the input x and its member linears (one member each when not grouped)."""
+    calls = []
+    for L in range(layers):
+        lin = {}
+        for (_, pi, name, rows, cols) in layer_shapes(1):
+            seed = synth.weight_seed("stack", L, pi)
+            R = synth.student_t_weight(rows, cols, seed, device=dev)
+            U, W = F.convert(R)
+            del R
+            codes, scales = F.quantize(U, W, T_STAGES)
+            del U, W
+            y = torch.empty((B, rows), dtype=torch.float32, device=dev)
+            lin[name] = dict(L=L, name=name, seed=seed, rows=rows, cols=cols, codes=codes,
+                             scales=scales, y=y)
+        groups = GROUPS if grouped else tuple((nm,) for g in GROUPS for nm in g)
+        for g in groups:
+            first = lin[g[0]]
+            x = synth.outlier_activations(B, first["cols"], synth.activation_seed(first["seed"], B),
+                                          device=dev)
+            calls.append(dict(x=x, rows=first["rows"], cols=first["cols"],
+                              members=[lin[nm] for nm in g]))
     torch.cuda.synchronize()
     status = F.get_status()
     if status != 0:
         raise RuntimeError(f"quantize status {status}")
-    return stack
+    return calls
+
+
+def call_bytes(c, B):
+    """Algorithmic bytes of one call: every member's codes, scales and y, the shared x once."""
+    per = [layer_bytes(m["rows"], m["cols"], B) for m in c["members"]]
+    return sum(per) - (len(per) - 1) * B * c["cols"] * 2
+
+
+def run_call(F, c):
+    if len(c["members"]) == 1:
+        m = c["members"][0]
+        F.wl_matmul(c["x"], m["codes"], m["scales"], c["rows"], y=m["y"])
+    else:
+        F.wl_matmul_group(c["x"], [m["codes"] for m in c["members"]],
+                          [m["scales"] for m in c["members"]], c["rows"],
+                          ys=[m["y"] for m in c["members"]])
 
 
 def run_ours(args, world, rank, local):
@@ -186,13 +215,15 @@ def run_ours(args, world, rank, local):
     F.load()
     dev = torch.device("cuda", local)
     B = args.batch
-    stack = build_stack(F, args.layers, B, dev)
-    step_bytes = sum(layer_bytes(s["rows"], s["cols"], B) for s in stack)
-    launches_per_step = len(stack)
+    calls = build_stack(F, args.layers, B, dev, grouped=not args.ungrouped)
+    step_bytes = sum(call_bytes(c, B) for c in calls)
+    nlinears = sum(len(c["members"]) for c in calls)
+    # a grouped call is one launch where the decode kernel takes it (B <= 2), else one per member
+    launches_per_step = len(calls) if B <= 2 else nlinears
 
     def step():
-        for s in stack:
-            F.wl_matmul(s["x"], s["codes"], s["scales"], s["rows"], y=s["y"])
+        for c in calls:
+            run_call(F, c)
 
     stream = torch.cuda.Stream(device=dev)
     with torch.cuda.stream(stream):
@@ -237,17 +268,18 @@ def run_ours(args, world, rank, local):
 
     # end to end through the public call with host buffers: per step the inputs of all
     # linears go host->device from pinned memory and every output comes back to the host.
-    xs_host = [s["x"].cpu().pin_memory() for s in stack]
-    ys_host = [torch.empty(s["y"].shape, dtype=torch.float32).pin_memory() for s in stack]
+    xs_host = [c["x"].cpu().pin_memory() for c in calls]
+    ys_dev = [m["y"] for c in calls for m in c["members"]]
+    ys_host = [torch.empty(y.shape, dtype=torch.float32).pin_memory() for y in ys_dev]
     h2d = sum(x.numel() * x.element_size() for x in xs_host)
     d2h = sum(y.numel() * 4 for y in ys_host)
 
     def e2e_step():
-        for s, xh in zip(stack, xs_host):
-            s["x"].copy_(xh, non_blocking=True)
+        for c, xh in zip(calls, xs_host):
+            c["x"].copy_(xh, non_blocking=True)
         run()
-        for s, yh in zip(stack, ys_host):
-            yh.copy_(s["y"], non_blocking=True)
+        for y, yh in zip(ys_dev, ys_host):
+            yh.copy_(y, non_blocking=True)
 
     with torch.cuda.stream(stream):
         for _ in range(args.warmup):
@@ -277,7 +309,9 @@ def run_ours(args, world, rank, local):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
         "data": "synthetic (seeded Student-t weights, N(0,1) bf16 activations with 1% x20 "
                 "outlier channels)",
-        "config": {"workload": WORKLOAD, "layers": args.layers, "linears": len(stack),
+        "config": {"workload": WORKLOAD, "layers": args.layers, "linears": nlinears,
+                   "calls_per_step": launches_per_step,
+                   "grouping": "none" if args.ungrouped else "qkv, o, gate+up, down (shared x)",
                    "T": T_STAGES, "batch": B, "x_dtype": "bf16",
                    "bytes_per_step": step_bytes, "cuda_graph": graph is not None,
                    "l2": "inputs larger than L2 (packed codes per step >> 129 MB)",
@@ -293,7 +327,7 @@ def run_ours(args, world, rank, local):
         "clocks": clk,
     }
     if not args.no_prefill:
-        del stack
+        del calls, ys_dev
         torch.cuda.empty_cache()
         line["prefill"] = run_prefill(F, dev, args.prefill_steps, max(args.warmup, 3))
     if rank == 0 and not args.no_cpu_baseline:
@@ -454,6 +488,7 @@ def main():
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--ref-linears", type=int, default=2)
     ap.add_argument("--no-prefill", action="store_true")
+    ap.add_argument("--ungrouped", action="store_true")
     ap.add_argument("--prefill-steps", type=int, default=10)
     args = ap.parse_args()
     world, rank, local = dist_setup()

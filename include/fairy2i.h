@@ -168,6 +168,24 @@ fairy2i_status fairy2i_wl_matmul_path(const void* x, fairy2i_dtype xdt, int64_t 
                                       float* y, int64_t ldy, int path, void* stream);
 
 /* ------------------------------------------------------------------------------------------
+ * Several linears of the same shape applied to the same input, e.g. the q, k, v projections
+ * or the gate and up projections of a decoder layer: for g < count,
+ *   y[g] = fairy2i_wl_matmul(x, xdt, B, in_features, ldx, codes[g], scales[g], out_features, T)
+ * with codes[g], scales[g], y[g] device pointers passed in host arrays of `count` entries
+ * (1 <= count <= FAIRY2I_MAX_GROUP). Where the decode kernel applies (B <= 2 bf16 tokens,
+ * T <= 4) the whole group is one launch; otherwise the members run one after the other on the
+ * automatic path. Requirements and errors are those of fairy2i_wl_matmul for every member
+ * (checked before anything is enqueued); FAIRY2I_ERR_INVALID_ARG for a count out of range or
+ * a null array. Results are bit-identical to the separate calls.
+ * ------------------------------------------------------------------------------------------ */
+#define FAIRY2I_MAX_GROUP 4
+fairy2i_status fairy2i_wl_matmul_group(const void* x, fairy2i_dtype xdt, int64_t B,
+                                       int64_t in_features, int64_t ldx, int count,
+                                       const uint32_t* const* codes, const float* const* scales,
+                                       int64_t out_features, int T, float* const* y, int64_t ldy,
+                                       void* stream);
+
+/* ------------------------------------------------------------------------------------------
  * Synchronizes `stream`, then returns and clears the device-side status of the current
  * device: FAIRY2I_ERR_NONFINITE, FAIRY2I_ERR_TIMEOUT, FAIRY2I_ERR_CUDA (an asynchronous CUDA
  * error) or FAIRY2I_OK.

@@ -35,7 +35,10 @@ SIGNATURES = {
     "fairy2i_get_status": ([_vp], _int),
     "fairy2i_quantize_noalloc": ([_vp, _vp, _i64, _i64, _i64, _int, _vp, _vp, _vp], _int),
     "fairy2i_selftest_wait_timeout": ([_c.c_uint32, _vp], _int),
+    "fairy2i_wl_matmul_group": ([_vp, _int, _i64, _i64, _i64, _int, _vp, _vp, _i64, _int, _vp,
+                                 _i64, _vp], _int),
 }
+MAX_GROUP = 4
 
 
 class Fairy2iError(RuntimeError):
@@ -145,6 +148,35 @@ def wl_matmul(x: torch.Tensor, codes: torch.Tensor, scales: torch.Tensor, out_fe
                                          _ptr(scales), out_features, T, _ptr(y), y.stride(0),
                                          path, _stream(stream)))
     return y
+
+
+def wl_matmul_group(x: torch.Tensor, codes, scales, out_features: int, ys=None, stream=None,
+                    T: int | None = None):
+    """Several linears of the same shape on one input x (CUDA): returns [y_g] with
+    y_g = wl_matmul(x, codes[g], scales[g], out_features); one launch where the decode kernel
+    applies."""
+    assert x.is_cuda and x.dim() == 2 and x.stride(1) == 1 and x.dtype in (torch.float32,
+                                                                          torch.bfloat16)
+    count = len(codes)
+    assert count == len(scales) and 1 <= count <= MAX_GROUP
+    B, in_features = x.shape
+    if T is None:
+        T = scales[0].shape[0]
+    if ys is None:
+        ys = [torch.empty((B, out_features), dtype=torch.float32, device=x.device)
+              for _ in range(count)]
+    assert len(ys) == count and all(y.stride(0) == ys[0].stride(0) for y in ys)
+    arr = ctypes.c_void_p * count
+    cp = arr(*[c.data_ptr() for c in codes])
+    sp = arr(*[s.data_ptr() for s in scales])
+    yp = arr(*[y.data_ptr() for y in ys])
+    xdt = F32 if x.dtype == torch.float32 else BF16
+    _check("fairy2i_wl_matmul_group",
+           load().fairy2i_wl_matmul_group(_ptr(x), xdt, B, in_features, x.stride(0), count,
+                                          ctypes.cast(cp, _vp), ctypes.cast(sp, _vp),
+                                          out_features, T, ctypes.cast(yp, _vp), ys[0].stride(0),
+                                          _stream(stream)))
+    return ys
 
 
 def selftest_wait_timeout(limit_us: int, stream=None):

@@ -30,6 +30,12 @@ fairy2i_status launch_wl_prefill(const void* x, fairy2i_dtype xdt, int64_t B, in
                                  int64_t n, int64_t m, int64_t out_features, int64_t wpr, int T,
                                  float* y, int64_t ldy, cudaStream_t stream, bool* handled);
 fairy2i_status launch_selftest_wait(uint32_t limit_us, cudaStream_t stream);
+fairy2i_status launch_wl_decode_group(const void* x, fairy2i_dtype xdt, int64_t B,
+                                      int64_t in_features, int64_t ldx, int count,
+                                      const uint32_t* const* codes, const float* const* scales,
+                                      int64_t n, int64_t m, int64_t out_features, int64_t wpr,
+                                      int T, float* const* y, int64_t ldy, cudaStream_t stream,
+                                      bool* handled);
 
 // Status word: one __device__ word per device that has loaded the module; its address is
 // looked up once per device with that device current.
@@ -151,6 +157,43 @@ fairy2i_status fairy2i_wl_matmul(const void* x, fairy2i_dtype xdt, int64_t B, in
                                  void* stream) {
   return fairy2i_wl_matmul_path(x, xdt, B, in_features, ldx, codes, scales, out_features, T, y,
                                 ldy, 0, stream);
+}
+
+fairy2i_status fairy2i_wl_matmul_group(const void* x, fairy2i_dtype xdt, int64_t B,
+                                       int64_t in_features, int64_t ldx, int count,
+                                       const uint32_t* const* codes, const float* const* scales,
+                                       int64_t out_features, int T, float* const* y, int64_t ldy,
+                                       void* stream) {
+  if (count < 1 || count > FAIRY2I_MAX_GROUP || !codes || !scales || !y)
+    return FAIRY2I_ERR_INVALID_ARG;
+  // Every member is validated as a single call would be (B = 0 included) before anything runs.
+  for (int g = 0; g < count; ++g) {
+    if (B < 0 || in_features < 1 || out_features < 1 || T < 1 || T > FAIRY2I_MAX_STAGES)
+      return FAIRY2I_ERR_INVALID_ARG;
+    if (xdt != FAIRY2I_F32 && xdt != FAIRY2I_BF16) return FAIRY2I_ERR_DTYPE;
+    if (B == 0) return FAIRY2I_OK;
+    if (!x || !codes[g] || !scales[g] || !y[g]) return FAIRY2I_ERR_INVALID_ARG;
+    if (ldx < in_features || ldy < out_features) return FAIRY2I_ERR_SHAPE;
+    if (!aligned(x, 16) || !aligned(codes[g], 16) || !aligned(y[g], 4) || !aligned(scales[g], 4))
+      return FAIRY2I_ERR_ALIGNMENT;
+  }
+  const int64_t n = (out_features + 1) / 2, m = (in_features + 1) / 2;
+  const int64_t wpr = fairy2i_codes_words_per_row(m);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  bool handled = false;
+  if (B <= 2) {   // one launch of the decode kernel for the whole group
+    const fairy2i_status st = launch_wl_decode_group(x, xdt, B, in_features, ldx, count, codes,
+                                                     scales, n, m, out_features, wpr, T, y, ldy,
+                                                     s, &handled);
+    if (handled || st != FAIRY2I_OK) return st;
+  }
+  for (int g = 0; g < count; ++g) {   // elsewhere: the automatic path per member
+    const fairy2i_status st = fairy2i_wl_matmul_path(x, xdt, B, in_features, ldx, codes[g],
+                                                     scales[g], out_features, T, y[g], ldy, 0,
+                                                     stream);
+    if (st != FAIRY2I_OK) return st;
+  }
+  return FAIRY2I_OK;
 }
 
 fairy2i_status fairy2i_selftest_wait_timeout(uint32_t limit_us, void* stream) {

@@ -53,15 +53,19 @@ constexpr int kMaxChunksPerWarp = 8;
 constexpr uint32_t kWaitLimit = 1u << 22;
 constexpr int kMaxSmem = 200 * 1024;
 
+constexpr int kMaxGroup = 4;                 // linears of one launch that share x
+
 struct Args {
-  const uint32_t* codes;
+  const uint32_t* codes[kMaxGroup];      // per linear of the group (same shape, same x)
+  const float* scales[kMaxGroup];
+  float* y[kMaxGroup];
   const __nv_bfloat16* x;
   int64_t B, in_features, ldx;
-  const float* scales;
   int64_t n, m, out_features, ldy;
   int wpr, nchunks;
+  int tiles;             // 16-row tiles per linear: CTA blockIdx.x works on linear
+                         // blockIdx.x / tiles, row tile blockIdx.x % tiles
   int x_vec;             // x rows 16-byte aligned with m % 8 == 0: vector loads allowed
-  float* y;
   unsigned int* status;
   int x_off, raw_off, red_off, bar_off, cpw;
 };
@@ -145,7 +149,10 @@ __global__ void __launch_bounds__(kThreads, 1) wl_decode_fp8_kernel(const Args a
   extern __shared__ __align__(1024) unsigned char smem[];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int g = lane >> 2, t4 = lane & 3;
-  const int64_t j0 = (int64_t)blockIdx.x * kRows;
+  const int lin = (int)blockIdx.x / a.tiles, tile = (int)blockIdx.x - lin * a.tiles;
+  const uint32_t* const codes = a.codes[lin];
+  const float* const scales = a.scales[lin];
+  const int64_t j0 = (int64_t)tile * kRows;
   const uint32_t* codes_s = reinterpret_cast<const uint32_t*>(smem);
   uint64_t* bar = reinterpret_cast<uint64_t*>(smem + a.bar_off) + warp;
   unsigned char* xw = smem + a.x_off + (size_t)warp * a.cpw * NB * kXBytes;
@@ -167,7 +174,7 @@ __global__ void __launch_bounds__(kThreads, 1) wl_decode_fp8_kernel(const Args a
 #pragma unroll
       for (int tm = 0; tm < T2; ++tm)
         bulk_load(smem + (size_t)(tm * a.nchunks + c_begin) * kTileBytes,
-                  a.codes + ((tm * tiles + blockIdx.x) * a.nchunks + c_begin) * kTileWords,
+                  codes + ((tm * tiles + tile) * a.nchunks + c_begin) * kTileWords,
                   (uint32_t)(nc * kTileBytes), bar);
     }
   }
@@ -304,8 +311,8 @@ __global__ void __launch_bounds__(kThreads, 1) wl_decode_fp8_kernel(const Args a
   float sre_u = 0.f, sre_w = 0.f;
 #pragma unroll
   for (int t = 0; t < T; ++t) {
-    sre_u += __ldg(a.scales + (t * 2 + 0) * 2);
-    sre_w += __ldg(a.scales + (t * 2 + 1) * 2);
+    sre_u += __ldg(scales + (t * 2 + 0) * 2);
+    sre_w += __ldg(scales + (t * 2 + 1) * 2);
   }
 #pragma unroll
   for (int b = 0; b < NB; ++b) {
@@ -315,8 +322,8 @@ __global__ void __launch_bounds__(kThreads, 1) wl_decode_fp8_kernel(const Args a
 #pragma unroll
     for (int tm = 0; tm < T2; ++tm) {
       const int t = tm >> 1, mat = tm & 1;
-      const float hr = 0.5f * __ldg(a.scales + (t * 2 + mat) * 2 + 0);
-      const float hs = 0.5f * __ldg(a.scales + (t * 2 + mat) * 2 + 1);
+      const float hr = 0.5f * __ldg(scales + (t * 2 + mat) * 2 + 0);
+      const float hs = 0.5f * __ldg(scales + (t * 2 + mat) * 2 + 1);
       const float hi = is_q ? -hs : hs;          // conj(h) multiplies Q
       const float di0 = mat ? -acc[b][tm][1] : acc[b][tm][1];   // W multiplies conj(x)
       const float di1 = mat ? -acc[b][tm][3] : acc[b][tm][3];
@@ -349,7 +356,7 @@ __global__ void __launch_bounds__(kThreads, 1) wl_decode_fp8_kernel(const Args a
     for (int w = 0; w < kWarps; ++w) sum += red[((w * NB + b) * kRows + r) * 2 + comp];
     const int64_t j = j0 + r;
     if (ok && j < a.n && b < a.B) {
-      float* yb = a.y + (int64_t)b * a.ldy;
+      float* yb = a.y[lin] + (int64_t)b * a.ldy;
       if (comp == 0) yb[j] = sum;
       else if (a.n + j < a.out_features) yb[a.n + j] = sum;
     }
@@ -376,7 +383,7 @@ inline Layout layout(int nchunks, int T, int NB) {
 }
 
 template <int NB, int T>
-fairy2i_status launch(Args a, const Layout& L, cudaStream_t stream) {
+fairy2i_status launch(Args a, int count, const Layout& L, cudaStream_t stream) {
   auto kern = wl_decode_fp8_kernel<NB, T>;
   static bool configured = false;
   if (!configured) {
@@ -386,7 +393,7 @@ fairy2i_status launch(Args a, const Layout& L, cudaStream_t stream) {
     configured = true;
   }
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)((a.n + kRows - 1) / kRows));
+  cfg.gridDim = dim3((unsigned)(a.tiles * count));
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = L.total;
   cfg.stream = stream;
@@ -401,40 +408,56 @@ fairy2i_status launch(Args a, const Layout& L, cudaStream_t stream) {
 
 }  // namespace dec
 
-fairy2i_status launch_wl_decode(const void* x, fairy2i_dtype xdt, int64_t B, int64_t in_features,
-                                int64_t ldx, const uint32_t* codes, const float* scales,
-                                int64_t n, int64_t m, int64_t out_features, int64_t wpr, int T,
-                                float* y, int64_t ldy, cudaStream_t stream, bool* handled) {
+// `count` linears of the same shape sharing x (codes[g], scales[g] -> y[g]) in one launch.
+fairy2i_status launch_wl_decode_group(const void* x, fairy2i_dtype xdt, int64_t B,
+                                      int64_t in_features, int64_t ldx, int count,
+                                      const uint32_t* const* codes, const float* const* scales,
+                                      int64_t n, int64_t m, int64_t out_features, int64_t wpr,
+                                      int T, float* const* y, int64_t ldy, cudaStream_t stream,
+                                      bool* handled) {
   using namespace dec;
   *handled = false;
-  if (xdt != FAIRY2I_BF16 || B > 2 || T > 4) return FAIRY2I_OK;
+  if (xdt != FAIRY2I_BF16 || B > 2 || T > 4 || count < 1 || count > kMaxGroup) return FAIRY2I_OK;
   const int nchunks = (int)(wpr / kChunkWords);
   const int NB = B > 1 ? 2 : 1;
   const Layout L = layout(nchunks, T, NB);
   if (L.total > kMaxSmem || m > (1 << 24) || (nchunks + kWarps - 1) / kWarps > kMaxChunksPerWarp)
     return FAIRY2I_OK;
   Args a;
-  a.codes = codes;
+  for (int g = 0; g < kMaxGroup; ++g) {
+    a.codes[g] = codes[g < count ? g : 0];
+    a.scales[g] = scales[g < count ? g : 0];
+    a.y[g] = y[g < count ? g : 0];
+  }
   a.x = reinterpret_cast<const __nv_bfloat16*>(x);
-  a.B = B; a.in_features = in_features; a.ldx = ldx; a.scales = scales;
+  a.B = B; a.in_features = in_features; a.ldx = ldx;
   a.n = n; a.m = m; a.out_features = out_features; a.ldy = ldy;
-  a.wpr = (int)wpr; a.nchunks = nchunks; a.y = y; a.status = device_status_word();
+  a.wpr = (int)wpr; a.nchunks = nchunks; a.status = device_status_word();
+  a.tiles = (int)((n + kRows - 1) / kRows);
   a.x_off = L.x_off; a.raw_off = L.raw_off; a.red_off = L.red_off; a.bar_off = L.bar_off;
   a.cpw = (nchunks + kWarps - 1) / kWarps;
   a.x_vec = (reinterpret_cast<uintptr_t>(x) % 16 == 0) && (ldx % 8 == 0) && (m % 8 == 0);
   *handled = true;
   switch (T * 4 + NB) {
-    case 1 * 4 + 1: return launch<1, 1>(a, L, stream);
-    case 1 * 4 + 2: return launch<2, 1>(a, L, stream);
-    case 2 * 4 + 1: return launch<1, 2>(a, L, stream);
-    case 2 * 4 + 2: return launch<2, 2>(a, L, stream);
-    case 3 * 4 + 1: return launch<1, 3>(a, L, stream);
-    case 3 * 4 + 2: return launch<2, 3>(a, L, stream);
-    case 4 * 4 + 1: return launch<1, 4>(a, L, stream);
-    case 4 * 4 + 2: return launch<2, 4>(a, L, stream);
+    case 1 * 4 + 1: return launch<1, 1>(a, count, L, stream);
+    case 1 * 4 + 2: return launch<2, 1>(a, count, L, stream);
+    case 2 * 4 + 1: return launch<1, 2>(a, count, L, stream);
+    case 2 * 4 + 2: return launch<2, 2>(a, count, L, stream);
+    case 3 * 4 + 1: return launch<1, 3>(a, count, L, stream);
+    case 3 * 4 + 2: return launch<2, 3>(a, count, L, stream);
+    case 4 * 4 + 1: return launch<1, 4>(a, count, L, stream);
+    case 4 * 4 + 2: return launch<2, 4>(a, count, L, stream);
   }
   *handled = false;
   return FAIRY2I_OK;
+}
+
+fairy2i_status launch_wl_decode(const void* x, fairy2i_dtype xdt, int64_t B, int64_t in_features,
+                                int64_t ldx, const uint32_t* codes, const float* scales,
+                                int64_t n, int64_t m, int64_t out_features, int64_t wpr, int T,
+                                float* y, int64_t ldy, cudaStream_t stream, bool* handled) {
+  return launch_wl_decode_group(x, xdt, B, in_features, ldx, 1, &codes, &scales, n, m,
+                                out_features, wpr, T, &y, ldy, stream, handled);
 }
 
 }  // namespace fairy2i

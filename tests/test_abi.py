@@ -99,3 +99,23 @@ def test_selftest_wait_timeout_validation(lib):
     """Out-of-range limits are refused before anything is enqueued."""
     assert lib.fairy2i_selftest_wait_timeout(0, None) == 1
     assert lib.fairy2i_selftest_wait_timeout(100001, None) == 1
+
+
+def test_wl_matmul_group_validation(lib):
+    arr = ctypes.c_void_p * 4
+
+    def call(count=3, B=1, inf=16, ldx=16, outf=16, T=2, ldy=16, xdt=1, codes=None, ys=None,
+             null_arrays=False):
+        cp = arr(*([GOOD] * 4)) if codes is None else codes
+        sp = arr(*([GOOD] * 4))
+        yp = arr(*([GOOD] * 4)) if ys is None else ys
+        if null_arrays:
+            cp = sp = yp = None
+        return lib.fairy2i_wl_matmul_group(GOOD, xdt, B, inf, ldx, count, cp, sp, outf, T, yp,
+                                           ldy, None)
+    assert call(B=0) == 0                                    # empty batch: nothing to do
+    assert call(count=0) == 1 and call(count=5) == 1 and call(null_arrays=True) == 1
+    assert call(T=0) == 1 and call(xdt=7) == 4
+    assert call(ldx=15) == 2 and call(ldy=15) == 2
+    assert call(codes=arr(GOOD, ODD, GOOD, GOOD)) == 3        # a misaligned member
+    assert call(ys=arr(GOOD, GOOD, None, GOOD)) == 1          # a null member

@@ -435,3 +435,32 @@ def test_bounded_wait_latches_timeout_and_context_survives(F):
     yg = _run_wl(F, x, codes, scales, 2 * n)
     xo = x.numpy()
     assert_wl_close(yg, O.wl_matmul(xo, codes, scales, 2 * n), xo, scales)
+
+
+# ------------------------------------------------------------------------------ grouped linears
+@pytest.mark.parametrize("out_f,in_f,T,B,count,dtype", [
+    (256, 512, 2, 1, 3, torch.bfloat16),      # one grouped decode launch (q, k, v shape class)
+    (130, 258, 3, 2, 2, torch.bfloat16),      # ragged rows, two tokens
+    (4096, 4096, 2, 1, 3, torch.bfloat16),    # the 7B attention projections
+    (11008, 4096, 2, 1, 2, torch.bfloat16),   # the 7B gate and up projections
+    (64, 256, 2, 5, 2, torch.bfloat16),       # B > 2: members on the prefill path
+    (37, 53, 2, 1, 4, torch.float32),         # fp32 x: members on the general path
+])
+def test_wl_matmul_group_equals_separate_calls(F, out_f, in_f, T, B, count, dtype):
+    """A group of linears on one input gives, bit for bit, the separate calls' results, and
+    every member matches the oracle."""
+    n, m = O.complex_dims(out_f, in_f)
+    layers = [_random_quantized(n, m, T, seed=41 + 7 * g + out_f) for g in range(count)]
+    x = synth.outlier_activations(B, in_f, seed=43 + in_f).to(dtype)
+    xd = x.to(DEV)
+    cds = [upload_codes(O.pack_codes(c)) for c, _ in layers]
+    scs = [torch.from_numpy(s).to(DEV) for _, s in layers]
+    ys = F.wl_matmul_group(xd, cds, scs, out_f)
+    singles = [F.wl_matmul(xd, c, s, out_f) for c, s in zip(cds, scs)]
+    assert F.get_status() == 0
+    xo = x.float().numpy()
+    for g, (yg, ys1) in enumerate(zip(ys, singles)):
+        assert torch.equal(yg, ys1)
+        if out_f * in_f <= 4096 * 4096 and g == 0:
+            codes, scales = layers[g]
+            assert_wl_close(yg.cpu().numpy(), O.wl_matmul(xo, codes, scales, out_f), xo, scales)
