@@ -54,9 +54,11 @@ def peaks():
 
 # DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) from ncu captures of the current
 # kernels (profiles/wl_decode_fp8_llama2_7b_stack_b1.md, profiles/wl_prefill_llama2_7b_2048tok.md):
-# one decoder layer's seven decode launches (every layer has the same shapes), and one T = 2
-# prefill launch of the 4096 -> 11008 layer on 2048 tokens.
-DECODE_DRAM_BYTES_PER_LAYER = 4 * 4.231e6 + 2 * 11.309e6 + 11.323e6
+# one decoder layer's decode launches (every layer has the same shapes; grouped: q/k/v, o,
+# gate/up, down; ungrouped: seven), and one T = 2 prefill launch of the 4096 -> 11008 layer on
+# 2048 tokens.
+DECODE_DRAM_BYTES_PER_LAYER = 12.621e6 + 4.232e6 + 22.582e6 + 11.323e6
+DECODE_DRAM_BYTES_PER_LAYER_UNGROUPED = 4 * 4.231e6 + 2 * 11.309e6 + 11.323e6
 PREFILL_T2_UP_DRAM_BYTES = 28.087e6 + 38.276e6
 
 PREFILL_TOKENS = 2048
@@ -321,7 +323,8 @@ def run_ours(args, world, rank, local):
         "gpu_launches": launches_per_step * args.steps,
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm,
                      "unit": "GB/s", "frac": round(achieved / hbm, 4),
-                     "traffic": int(DECODE_DRAM_BYTES_PER_LAYER * args.layers),
+                     "traffic": int((DECODE_DRAM_BYTES_PER_LAYER_UNGROUPED if args.ungrouped
+                                     else DECODE_DRAM_BYTES_PER_LAYER) * args.layers),
                      "peak_kind": f"{peak_kind} hbm_gbs (burst copy)",
                      "kernel": "wl_matmul decode (all launches of the step)"},
         "clocks": clk,
