@@ -37,7 +37,7 @@ __all__ = [
     "complex_dims", "convert", "realify_lin", "realify_conj", "project", "fixed_tree_sum",
     "axis_scales", "dequant", "residual_quantize", "quantize", "words_per_row", "row_tiles",
     "pack_codes", "unpack_codes", "split_input", "wl_matmul", "wl_matmul_rows", "dense_realified",
-    "tolerance_bound",
+    "tolerance_bound", "adjoint_codes",
 ]
 
 F32 = np.float32
@@ -320,6 +320,22 @@ def wl_matmul(x, codes, scales, out_features: int):
     n, m = np.shape(codes)[2], np.shape(codes)[3]
     y = wl_matmul_rows(split_input(x, m), codes, scales)
     return np.concatenate([y.real, y.imag], axis=1)[:, :out_features]
+
+
+def adjoint_codes(codes):
+    """Codes of the adjoint layer, whose real map is R^T (the input gradient of the quantized
+    layer, the straight-through backward of Sec. 3.2 / Sec. 3.3 for x).
+
+    From Eq. realify-ops: R_lin(U)^T = R_lin(U^H) and R_conj(W)^T = R_conj(W^T), so the transpose
+    of R^ = sum_t R_lin(U^(t)) + R_conj(W^(t)) (Eq. R-sum) is the widely-linear map with
+    U' = U^(t)H and W' = W^(t)T, both m x n. With U^ = s_re b_re + i s_im b_im (Eq.
+    ifairy-dequant), U^H holds conj(b) = i^(-c) with the same scales: the U codes are transposed
+    and conjugated (c -> (4 - c) mod 4), the W codes transposed; the scales do not change.
+    codes [T][2][n][m] -> [T][2][m][n]."""
+    codes = np.asarray(codes)
+    out = np.ascontiguousarray(np.transpose(codes, (0, 1, 3, 2))).astype(np.int64)
+    out[:, 0] = (4 - out[:, 0]) % 4
+    return out.astype(codes.dtype)
 
 
 def dense_realified(codes, scales):

@@ -350,3 +350,41 @@ def test_tolerance_bound_bounds_y():
     n = 32
     mag = np.abs(y[:, :n] + 1j * y[:, n:])
     assert np.all(mag.max(axis=1) <= O.tolerance_bound(x, scales) * (1 + 1e-12))
+
+
+# ------------------------------------------------------------------ adjoint (input gradient)
+@pytest.mark.parametrize("n,m,T", [(3, 5, 1), (4, 4, 2), (7, 2, 3), (1, 9, 2)])
+def test_adjoint_codes_realify_to_the_transpose(n, m, T):
+    """The adjoint codes realify (Eq. realify-ops, Eq. R-sum) to exactly the transpose of the
+    original layer's real map, for every code value in U and in W (a missing conjugation, a
+    conjugated W or an untransposed block fails)."""
+    g = np.random.default_rng(n * 31 + m * 7 + T)
+    codes = g.integers(0, 4, (T, 2, n, m)).astype(np.uint8)
+    scales = (0.01 + 0.03 * g.random((T, 2, 2))).astype(np.float32)
+    Rh = O.dense_realified(codes, scales)
+    Ra = O.dense_realified(O.adjoint_codes(codes), scales)
+    assert Ra.shape == (2 * m, 2 * n)
+    assert np.array_equal(Ra, Rh.T)
+
+
+def test_adjoint_codes_are_an_involution():
+    g = np.random.default_rng(5)
+    codes = g.integers(0, 4, (3, 2, 6, 11)).astype(np.uint8)
+    assert np.array_equal(O.adjoint_codes(O.adjoint_codes(codes)), codes)
+
+
+@pytest.mark.parametrize("out_f,in_f", [(6, 10), (7, 9), (9, 4)])
+def test_adjoint_matmul_is_the_input_gradient(out_f, in_f):
+    """<R^ x~, g~> = <x~, wl_matmul(g~, adjoint codes)> for the real layouts, odd sizes included
+    (the padded output channel carries no gradient)."""
+    g = np.random.default_rng(out_f + 10 * in_f)
+    n, m = O.complex_dims(out_f, in_f)
+    codes = g.integers(0, 4, (2, 2, n, m)).astype(np.uint8)
+    scales = (0.01 + 0.03 * g.random((2, 2, 2))).astype(np.float32)
+    x = g.standard_normal((3, in_f))
+    gy = g.standard_normal((3, out_f))
+    y = O.wl_matmul(x, codes, scales, out_f)
+    gx = O.wl_matmul(gy, O.adjoint_codes(codes), scales, in_f)
+    assert np.allclose(np.sum(y * gy, axis=1), np.sum(x * gx, axis=1), rtol=1e-12, atol=1e-12)
+    Rh = O.dense_realified(codes, scales)[:out_f, :in_f]
+    assert np.allclose(gx, gy @ Rh, rtol=1e-12, atol=1e-12)
