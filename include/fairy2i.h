@@ -168,6 +168,24 @@ fairy2i_status fairy2i_wl_matmul_path(const void* x, fairy2i_dtype xdt, int64_t 
                                       float* y, int64_t ldy, int path, void* stream);
 
 /* ------------------------------------------------------------------------------------------
+ * Codes of the adjoint layer: the input gradient of the quantized layer (the straight-through
+ * backward for x of Sec. 3.2/3.3), x~_grad = R^T y~_grad with R^ = sum_t R_lin(U^(t)) +
+ * R_conj(W^(t)). By Eq. realify-ops, R_lin(U)^T = R_lin(U^H) and R_conj(W)^T = R_conj(W^T), so
+ * the adjoint is the widely-linear layer U' = U^H, W' = W^T (m x n): the code matrices are
+ * transposed, the U codes conjugated (+i <-> -i), and the scales are unchanged. Then
+ *   fairy2i_wl_matmul(y_grad, dtype, B, out_features, ldg, codes_adj, scales, in_features, T,
+ *                     x_grad, ldxg, stream)
+ * computes x~_grad for y~_grad [B][out_features] (the padded output channel of an odd
+ * out_features carries no gradient, matching the zero padding of the input).
+ *   codes      as written by fairy2i_quantize for (n, m, T): fairy2i_codes_words(n, m, T) words.
+ *   codes_adj  fairy2i_codes_words(m, n, T) words, written completely (padding codes 0); must
+ *              not overlap codes.
+ *   Requirements: n, m >= 1, 1 <= T <= 8, both buffers 16-byte aligned.
+ * ------------------------------------------------------------------------------------------ */
+fairy2i_status fairy2i_codes_adjoint(const uint32_t* codes, int64_t n, int64_t m, int T,
+                                     uint32_t* codes_adj, void* stream);
+
+/* ------------------------------------------------------------------------------------------
  * Several linears of the same shape applied to the same input, e.g. the q, k, v projections
  * or the gate and up projections of a decoder layer: for g < count,
  *   y[g] = fairy2i_wl_matmul(x, xdt, B, in_features, ldx, codes[g], scales[g], out_features, T)

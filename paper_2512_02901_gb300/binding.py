@@ -37,6 +37,7 @@ SIGNATURES = {
     "fairy2i_selftest_wait_timeout": ([_c.c_uint32, _vp], _int),
     "fairy2i_wl_matmul_group": ([_vp, _int, _i64, _i64, _i64, _int, _vp, _vp, _i64, _int, _vp,
                                  _i64, _vp], _int),
+    "fairy2i_codes_adjoint": ([_vp, _i64, _i64, _int, _vp, _vp], _int),
 }
 MAX_GROUP = 4
 
@@ -177,6 +178,16 @@ def wl_matmul_group(x: torch.Tensor, codes, scales, out_features: int, ys=None, 
                                           out_features, T, ctypes.cast(yp, _vp), ys[0].stride(0),
                                           _stream(stream)))
     return ys
+
+
+def codes_adjoint(codes: torch.Tensor, n: int, m: int, T: int, stream=None) -> torch.Tensor:
+    """Codes of the adjoint layer (input gradient, R^T): the layout fairy2i_quantize writes for
+    an m x n layer. wl_matmul(y_grad, codes_adjoint(...), scales, in_features) = x~_grad."""
+    out = torch.empty(int(load().fairy2i_codes_words(m, n, T)), dtype=torch.int32,
+                      device=codes.device)
+    _check("fairy2i_codes_adjoint",
+           load().fairy2i_codes_adjoint(_ptr(codes), n, m, T, _ptr(out), _stream(stream)))
+    return out
 
 
 def selftest_wait_timeout(limit_us: int, stream=None):

@@ -30,6 +30,8 @@ fairy2i_status launch_wl_prefill(const void* x, fairy2i_dtype xdt, int64_t B, in
                                  int64_t n, int64_t m, int64_t out_features, int64_t wpr, int T,
                                  float* y, int64_t ldy, cudaStream_t stream, bool* handled);
 fairy2i_status launch_selftest_wait(uint32_t limit_us, cudaStream_t stream);
+fairy2i_status launch_codes_adjoint(const uint32_t* codes, int64_t n, int64_t m, int T,
+                                    uint32_t* codes_adj, cudaStream_t stream);
 fairy2i_status launch_wl_decode_group(const void* x, fairy2i_dtype xdt, int64_t B,
                                       int64_t in_features, int64_t ldx, int count,
                                       const uint32_t* const* codes, const float* const* scales,
@@ -194,6 +196,19 @@ fairy2i_status fairy2i_wl_matmul_group(const void* x, fairy2i_dtype xdt, int64_t
     if (st != FAIRY2I_OK) return st;
   }
   return FAIRY2I_OK;
+}
+
+fairy2i_status fairy2i_codes_adjoint(const uint32_t* codes, int64_t n, int64_t m, int T,
+                                     uint32_t* codes_adj, void* stream) {
+  if (!codes || !codes_adj || n < 1 || m < 1 || T < 1 || T > FAIRY2I_MAX_STAGES)
+    return FAIRY2I_ERR_INVALID_ARG;
+  if (n > (int64_t(1) << 40) / m) return FAIRY2I_ERR_SHAPE;
+  if (!aligned(codes, 16) || !aligned(codes_adj, 16)) return FAIRY2I_ERR_ALIGNMENT;
+  const uintptr_t a0 = reinterpret_cast<uintptr_t>(codes), b0 = reinterpret_cast<uintptr_t>(codes_adj);
+  const uintptr_t a1 = a0 + 4 * (uintptr_t)fairy2i_codes_words(n, m, T);
+  const uintptr_t b1 = b0 + 4 * (uintptr_t)fairy2i_codes_words(m, n, T);
+  if (a0 < b1 && b0 < a1) return FAIRY2I_ERR_INVALID_ARG;   // the buffers must not overlap
+  return launch_codes_adjoint(codes, n, m, T, codes_adj, static_cast<cudaStream_t>(stream));
 }
 
 fairy2i_status fairy2i_selftest_wait_timeout(uint32_t limit_us, void* stream) {

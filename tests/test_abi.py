@@ -119,3 +119,11 @@ def test_wl_matmul_group_validation(lib):
     assert call(ldx=15) == 2 and call(ldy=15) == 2
     assert call(codes=arr(GOOD, ODD, GOOD, GOOD)) == 3        # a misaligned member
     assert call(ys=arr(GOOD, GOOD, None, GOOD)) == 1          # a null member
+
+
+def test_codes_adjoint_validation(lib):
+    assert lib.fairy2i_codes_adjoint(None, 4, 4, 2, GOOD, None) == 1
+    assert lib.fairy2i_codes_adjoint(GOOD, 0, 4, 2, P((1 << 24)), None) == 1
+    assert lib.fairy2i_codes_adjoint(GOOD, 4, 4, 9, P((1 << 24)), None) == 1
+    assert lib.fairy2i_codes_adjoint(ODD, 4, 4, 2, P((1 << 24)), None) == 3
+    assert lib.fairy2i_codes_adjoint(GOOD, 4, 4, 2, GOOD, None) == 1     # overlapping buffers

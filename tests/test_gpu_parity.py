@@ -464,3 +464,34 @@ def test_wl_matmul_group_equals_separate_calls(F, out_f, in_f, T, B, count, dtyp
         if out_f * in_f <= 4096 * 4096 and g == 0:
             codes, scales = layers[g]
             assert_wl_close(yg.cpu().numpy(), O.wl_matmul(xo, codes, scales, out_f), xo, scales)
+
+
+# ------------------------------------------------------------------------------ adjoint (input gradient)
+@pytest.mark.parametrize("n,m,T", [(5, 9, 1), (16, 128, 2), (130, 300, 3), (257, 129, 4), (1, 1, 1),
+                                   (2048, 5504, 2)])
+def test_codes_adjoint_bit_exact(F, n, m, T):
+    """Transposed, U-conjugated codes in the packed layout of an m x n layer, bit for bit."""
+    codes, _ = _random_quantized(n, m, T, seed=n * 13 + m + T)
+    got = F.codes_adjoint(upload_codes(O.pack_codes(codes)), n, m, T)
+    assert F.get_status() == 0
+    want = O.pack_codes(O.adjoint_codes(codes))
+    assert np.array_equal(_np_codes(got), want)
+
+
+@pytest.mark.parametrize("out_f,in_f,T,B,dtype", [
+    (4096, 4096, 2, 1, torch.bfloat16),      # decode kernel on the adjoint codes
+    (129, 258, 3, 2, torch.bfloat16),
+    (64, 512, 2, 70, torch.bfloat16),        # prefill kernel
+    (37, 53, 2, 3, torch.float32),           # general kernel, odd sizes
+])
+def test_input_gradient_through_adjoint_codes(F, out_f, in_f, T, B, dtype):
+    """x~_grad = R^T y~_grad through the adjoint codes and the ordinary matmul paths."""
+    n, m = O.complex_dims(out_f, in_f)
+    codes, scales = _random_quantized(n, m, T, seed=out_f + 3 * in_f)
+    adj = F.codes_adjoint(upload_codes(O.pack_codes(codes)), n, m, T)
+    gy = synth.outlier_activations(B, out_f, seed=out_f * 5 + B).to(dtype)
+    gx = F.wl_matmul(gy.to(DEV), adj, torch.from_numpy(scales).to(DEV), in_f)
+    assert F.get_status() == 0
+    go = gy.float().numpy()
+    want = O.wl_matmul(go, O.adjoint_codes(codes), scales, in_f)
+    assert_wl_close(gx.cpu().numpy(), want, go, scales)
