@@ -61,6 +61,15 @@ DECODE_DRAM_BYTES_PER_LAYER = 12.621e6 + 4.232e6 + 22.582e6 + 11.323e6
 DECODE_DRAM_BYTES_PER_LAYER_UNGROUPED = 4 * 4.231e6 + 2 * 11.309e6 + 11.323e6
 PREFILL_T2_UP_DRAM_BYTES = 28.087e6 + 38.276e6
 
+def decode_traffic(args):
+    """ncu DRAM bytes of one step's decode launches, where a capture of the kernels this run
+    uses exists (the warp-MMA kernel on every call: --decode-path 1); else None."""
+    if args.decode_path != 1 or args.batch != 1:
+        return None
+    return int((DECODE_DRAM_BYTES_PER_LAYER_UNGROUPED if args.ungrouped
+                else DECODE_DRAM_BYTES_PER_LAYER) * args.layers)
+
+
 PREFILL_TOKENS = 2048
 PREFILL_LAYERS = (("up", 11008, 4096, 0), ("down", 4096, 11008, 1))   # (name, out, in, seed idx)
 
@@ -200,14 +209,14 @@ def call_bytes(c, B):
     return sum(per) - (len(per) - 1) * B * c["cols"] * 2
 
 
-def run_call(F, c):
+def run_call(F, c, path=0):
     if len(c["members"]) == 1:
         m = c["members"][0]
-        F.wl_matmul(c["x"], m["codes"], m["scales"], c["rows"], y=m["y"])
+        F.wl_matmul(c["x"], m["codes"], m["scales"], c["rows"], y=m["y"], path=path)
     else:
         F.wl_matmul_group(c["x"], [m["codes"] for m in c["members"]],
                           [m["scales"] for m in c["members"]], c["rows"],
-                          ys=[m["y"] for m in c["members"]])
+                          ys=[m["y"] for m in c["members"]], path=path)
 
 
 def run_ours(args, world, rank, local):
@@ -225,7 +234,7 @@ def run_ours(args, world, rank, local):
 
     def step():
         for c in calls:
-            run_call(F, c)
+            run_call(F, c, args.decode_path)
 
     stream = torch.cuda.Stream(device=dev)
     with torch.cuda.stream(stream):
@@ -314,6 +323,7 @@ def run_ours(args, world, rank, local):
         "config": {"workload": WORKLOAD, "layers": args.layers, "linears": nlinears,
                    "calls_per_step": launches_per_step,
                    "grouping": "none" if args.ungrouped else "qkv, o, gate+up, down (shared x)",
+                   "decode_path": args.decode_path,
                    "T": T_STAGES, "batch": B, "x_dtype": "bf16",
                    "bytes_per_step": step_bytes, "cuda_graph": graph is not None,
                    "l2": "inputs larger than L2 (packed codes per step >> 129 MB)",
@@ -323,8 +333,7 @@ def run_ours(args, world, rank, local):
         "gpu_launches": launches_per_step * args.steps,
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm,
                      "unit": "GB/s", "frac": round(achieved / hbm, 4),
-                     "traffic": int((DECODE_DRAM_BYTES_PER_LAYER_UNGROUPED if args.ungrouped
-                                     else DECODE_DRAM_BYTES_PER_LAYER) * args.layers),
+                     "traffic": decode_traffic(args),
                      "peak_kind": f"{peak_kind} hbm_gbs (burst copy)",
                      "kernel": "wl_matmul decode (all launches of the step)"},
         "clocks": clk,
@@ -493,6 +502,8 @@ def main():
     ap.add_argument("--no-prefill", action="store_true")
     ap.add_argument("--ungrouped", action="store_true")
     ap.add_argument("--prefill-steps", type=int, default=10)
+    ap.add_argument("--decode-path", type=int, default=0, choices=[0, 1, 4],
+                    help="decode kernel: 0 automatic, 1 warp-MMA, 4 persistent tcgen05")
     args = ap.parse_args()
     world, rank, local = dist_setup()
     if args.impl == "reference":

@@ -151,8 +151,9 @@ fairy2i_status fairy2i_wl_matmul(const void* x, fairy2i_dtype xdt, int64_t B,
                                  int64_t ldy, void* stream);
 
 /* Same as fairy2i_wl_matmul with the kernel chosen by `path`:
- *   0 = automatic: B <= 2 bf16 tokens and T <= 4 -> the warp-MMA decode kernel; B > 2 -> the
- *       tcgen05 prefill GEMM where it applies (see 3); otherwise the general CUDA-core kernel;
+ *   0 = automatic: B <= 2 bf16 tokens and T <= 4 -> a decode kernel: the persistent tcgen05 one
+ *       (4) when the call's 16-row tiles outnumber the SMs, else the warp-MMA one (1); B > 2 ->
+ *       the tcgen05 prefill GEMM where it applies (see 3); otherwise the general CUDA-core kernel;
  *   1 = the decode kernel where it applies, otherwise the general kernel;
  *   2 = the tcgen05 decode kernel (5th-generation tensor cores, the code matrix in tensor
  *       memory); it takes B <= 2 bf16 tokens, T <= 4 and rows of at most 176 128-code chunks
@@ -160,7 +161,16 @@ fairy2i_status fairy2i_wl_matmul(const void* x, fairy2i_dtype xdt, int64_t B,
  *   3 = the tcgen05 prefill GEMM (codes expanded into bf16 +-1 tiles in tensor memory, x by TMA,
  *       64 tokens per tile); it takes bf16 x with 16-byte aligned rows, ldx % 8 == 0,
  *       m % 8 == 0 (m = ceil(in_features/2)) and T <= 4, and returns FAIRY2I_ERR_INVALID_ARG for
+ *       anything else;
+ *   4 = the persistent tcgen05 decode kernel (one CTA per SM looping over row blocks, the codes
+ *       streamed through shared memory and decoded into tensor memory, K split over thread-block
+ *       clusters of up to 8 CTAs whose partial rows are summed in rank order); it takes B <= 2
+ *       bf16 tokens, T <= 4 and in_features <= 24576 and returns FAIRY2I_ERR_INVALID_ARG for
  *       anything else.
+ * The decode kernels (paths 1, 2, 4) read the codes and scales before waiting for the previous
+ * kernel in the stream (programmatic dependent launch): the codes must not be written by the
+ * kernel launched right before the matmul on the same stream unless that kernel is one of this
+ * library's convert/quantize/adjoint kernels, which end before any dependent kernel starts.
  * Results agree within the float32-accumulation tolerance whichever path runs. */
 fairy2i_status fairy2i_wl_matmul_path(const void* x, fairy2i_dtype xdt, int64_t B,
                                       int64_t in_features, int64_t ldx, const uint32_t* codes,
@@ -190,11 +200,14 @@ fairy2i_status fairy2i_codes_adjoint(const uint32_t* codes, int64_t n, int64_t m
  * or the gate and up projections of a decoder layer: for g < count,
  *   y[g] = fairy2i_wl_matmul(x, xdt, B, in_features, ldx, codes[g], scales[g], out_features, T)
  * with codes[g], scales[g], y[g] device pointers passed in host arrays of `count` entries
- * (1 <= count <= FAIRY2I_MAX_GROUP). Where the decode kernel applies (B <= 2 bf16 tokens,
- * T <= 4) the whole group is one launch; otherwise the members run one after the other on the
- * automatic path. Requirements and errors are those of fairy2i_wl_matmul for every member
- * (checked before anything is enqueued); FAIRY2I_ERR_INVALID_ARG for a count out of range or
- * a null array. Results are bit-identical to the separate calls.
+ * (1 <= count <= FAIRY2I_MAX_GROUP). Where a decode kernel applies (B <= 2 bf16 tokens,
+ * T <= 4) the whole group is one launch, of the persistent tcgen05 kernel when the group's 16-row
+ * tiles outnumber the SMs, else of the warp-MMA kernel; otherwise the members run one after the
+ * other on the automatic path. Requirements and errors are those of fairy2i_wl_matmul for every
+ * member (checked before anything is enqueued); FAIRY2I_ERR_INVALID_ARG for a count out of range
+ * or a null array. Results agree with the separate calls within the float32-accumulation
+ * tolerance (the kernel may differ: a group has more tiles than each member); on the warp-MMA
+ * kernel they are bit-identical.
  * ------------------------------------------------------------------------------------------ */
 #define FAIRY2I_MAX_GROUP 4
 fairy2i_status fairy2i_wl_matmul_group(const void* x, fairy2i_dtype xdt, int64_t B,
@@ -202,6 +215,19 @@ fairy2i_status fairy2i_wl_matmul_group(const void* x, fairy2i_dtype xdt, int64_t
                                        const uint32_t* const* codes, const float* const* scales,
                                        int64_t out_features, int T, float* const* y, int64_t ldy,
                                        void* stream);
+
+/* fairy2i_wl_matmul_group with the decode kernel chosen by `path`: 0 = automatic (as above),
+ * 1 = the warp-MMA decode kernel where it applies (else the automatic path per member),
+ * 4 = the persistent tcgen05 decode kernel, one launch for the group (B <= 2 bf16 tokens, T <= 4,
+ * in_features <= 24576; FAIRY2I_ERR_INVALID_ARG for anything else). Any other path returns
+ * FAIRY2I_ERR_INVALID_ARG. Results agree with the separate calls within the float32-accumulation
+ * tolerance (bit-identical for path 1). */
+fairy2i_status fairy2i_wl_matmul_group_path(const void* x, fairy2i_dtype xdt, int64_t B,
+                                            int64_t in_features, int64_t ldx, int count,
+                                            const uint32_t* const* codes,
+                                            const float* const* scales, int64_t out_features,
+                                            int T, float* const* y, int64_t ldy, int path,
+                                            void* stream);
 
 /* ------------------------------------------------------------------------------------------
  * Synchronizes `stream`, then returns and clears the device-side status of the current

@@ -12,7 +12,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libfairy2i.so")
 
 F32, BF16 = 0, 1
-PATH_AUTO, PATH_DECODE, PATH_TC_DECODE, PATH_TC_PREFILL = 0, 1, 2, 3
+PATH_AUTO, PATH_DECODE, PATH_TC_DECODE, PATH_TC_PREFILL, PATH_STREAM = 0, 1, 2, 3, 4
 MAX_STAGES = 8
 STATUS = {0: "ok", 1: "invalid argument", 2: "shape", 3: "alignment", 4: "dtype", 5: "workspace",
           6: "non-finite weight", 7: "device wait timeout", 8: "CUDA error"}
@@ -38,6 +38,8 @@ SIGNATURES = {
     "fairy2i_wl_matmul_group": ([_vp, _int, _i64, _i64, _i64, _int, _vp, _vp, _i64, _int, _vp,
                                  _i64, _vp], _int),
     "fairy2i_codes_adjoint": ([_vp, _i64, _i64, _int, _vp, _vp], _int),
+    "fairy2i_wl_matmul_group_path": ([_vp, _int, _i64, _i64, _i64, _int, _vp, _vp, _i64, _int,
+                                      _vp, _i64, _int, _vp], _int),
 }
 MAX_GROUP = 4
 
@@ -152,10 +154,10 @@ def wl_matmul(x: torch.Tensor, codes: torch.Tensor, scales: torch.Tensor, out_fe
 
 
 def wl_matmul_group(x: torch.Tensor, codes, scales, out_features: int, ys=None, stream=None,
-                    T: int | None = None):
+                    T: int | None = None, path: int = PATH_AUTO):
     """Several linears of the same shape on one input x (CUDA): returns [y_g] with
-    y_g = wl_matmul(x, codes[g], scales[g], out_features); one launch where the decode kernel
-    applies."""
+    y_g = wl_matmul(x, codes[g], scales[g], out_features); one launch where a decode kernel
+    applies (path 0 automatic, 1 the warp-MMA decode kernel, 4 the persistent tcgen05 one)."""
     assert x.is_cuda and x.dim() == 2 and x.stride(1) == 1 and x.dtype in (torch.float32,
                                                                           torch.bfloat16)
     count = len(codes)
@@ -172,11 +174,11 @@ def wl_matmul_group(x: torch.Tensor, codes, scales, out_features: int, ys=None, 
     sp = arr(*[s.data_ptr() for s in scales])
     yp = arr(*[y.data_ptr() for y in ys])
     xdt = F32 if x.dtype == torch.float32 else BF16
-    _check("fairy2i_wl_matmul_group",
-           load().fairy2i_wl_matmul_group(_ptr(x), xdt, B, in_features, x.stride(0), count,
-                                          ctypes.cast(cp, _vp), ctypes.cast(sp, _vp),
-                                          out_features, T, ctypes.cast(yp, _vp), ys[0].stride(0),
-                                          _stream(stream)))
+    _check("fairy2i_wl_matmul_group_path",
+           load().fairy2i_wl_matmul_group_path(_ptr(x), xdt, B, in_features, x.stride(0), count,
+                                               ctypes.cast(cp, _vp), ctypes.cast(sp, _vp),
+                                               out_features, T, ctypes.cast(yp, _vp),
+                                               ys[0].stride(0), path, _stream(stream)))
     return ys
 
 

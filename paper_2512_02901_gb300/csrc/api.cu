@@ -29,6 +29,12 @@ fairy2i_status launch_wl_prefill(const void* x, fairy2i_dtype xdt, int64_t B, in
                                  int64_t ldx, const uint32_t* codes, const float* scales,
                                  int64_t n, int64_t m, int64_t out_features, int64_t wpr, int T,
                                  float* y, int64_t ldy, cudaStream_t stream, bool* handled);
+fairy2i_status launch_wl_stream_group(const void* x, fairy2i_dtype xdt, int64_t B,
+                                      int64_t in_features, int64_t ldx, int count,
+                                      const uint32_t* const* codes, const float* const* scales,
+                                      int64_t n, int64_t m, int64_t out_features, int64_t wpr,
+                                      int T, float* const* y, int64_t ldy, cudaStream_t stream,
+                                      bool* handled);
 fairy2i_status launch_selftest_wait(uint32_t limit_us, cudaStream_t stream);
 fairy2i_status launch_codes_adjoint(const uint32_t* codes, int64_t n, int64_t m, int T,
                                     uint32_t* codes_adj, cudaStream_t stream);
@@ -58,6 +64,19 @@ unsigned int* device_status_word() {
 }
 
 static bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+// Automatic choice between the two decode kernels (B <= 2 bf16 tokens): the warp-MMA kernel
+// gives each 16-row tile its own CTA, so once the tiles of the call outnumber the SMs it runs in
+// several waves and the persistent tcgen05 kernel (one wave, every CTA looping over row blocks)
+// is faster; with at most one wave the warp-MMA kernel's shorter launch wins.
+static bool prefer_stream(int64_t n, int count) {
+  static int sms[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
+  if (!sms[dev] && cudaDeviceGetAttribute(&sms[dev], cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return false;
+  return (int64_t)count * ((n + 15) / 16) > sms[dev];
+}
 
 }  // namespace fairy2i
 
@@ -121,7 +140,7 @@ fairy2i_status fairy2i_wl_matmul_path(const void* x, fairy2i_dtype xdt, int64_t 
                                       const float* scales, int64_t out_features, int T, float* y,
                                       int64_t ldy, int path, void* stream) {
   if (B < 0 || in_features < 1 || out_features < 1 || T < 1 || T > FAIRY2I_MAX_STAGES ||
-      path < 0 || path > 3)
+      path < 0 || path > 4)
     return FAIRY2I_ERR_INVALID_ARG;
   if (xdt != FAIRY2I_F32 && xdt != FAIRY2I_BF16) return FAIRY2I_ERR_DTYPE;
   if (B == 0) return FAIRY2I_OK;
@@ -140,11 +159,22 @@ fairy2i_status fairy2i_wl_matmul_path(const void* x, fairy2i_dtype xdt, int64_t 
     if (handled || st != FAIRY2I_OK) return st;
     if (path == 3) return FAIRY2I_ERR_INVALID_ARG;   // outside the prefill kernel's domain
   }
+  if (path == 4) {   // persistent tcgen05 decode kernel (explicit): B <= 2 bf16 tokens, T <= 4
+    st = launch_wl_stream_group(x, xdt, B, in_features, ldx, 1, &codes, &scales, n, m,
+                                out_features, wpr, T, &y, ldy, s, &handled);
+    if (handled || st != FAIRY2I_OK) return st;
+    return FAIRY2I_ERR_INVALID_ARG;   // shape or dtype outside the kernel
+  }
   if (path == 2) {   // tcgen05 decode kernel (explicit): B <= 2 bf16 tokens, T <= 4
     st = launch_wl_tc(x, xdt, B, in_features, ldx, codes, scales, n, m, out_features, wpr, T, y,
                       ldy, s, &handled);
     if (handled || st != FAIRY2I_OK) return st;
     return FAIRY2I_ERR_INVALID_ARG;   // shape or dtype outside the tcgen05 decode kernel
+  }
+  if (path == 0 && B <= 2 && xdt == FAIRY2I_BF16 && prefer_stream(n, 1)) {
+    st = launch_wl_stream_group(x, xdt, B, in_features, ldx, 1, &codes, &scales, n, m,
+                                out_features, wpr, T, &y, ldy, s, &handled);
+    if (handled || st != FAIRY2I_OK) return st;
   }
   st = launch_wl_decode(x, xdt, B, in_features, ldx, codes, scales, n, m,
                                        out_features, wpr, T, y, ldy, s, &handled);
@@ -161,12 +191,14 @@ fairy2i_status fairy2i_wl_matmul(const void* x, fairy2i_dtype xdt, int64_t B, in
                                 ldy, 0, stream);
 }
 
-fairy2i_status fairy2i_wl_matmul_group(const void* x, fairy2i_dtype xdt, int64_t B,
-                                       int64_t in_features, int64_t ldx, int count,
-                                       const uint32_t* const* codes, const float* const* scales,
-                                       int64_t out_features, int T, float* const* y, int64_t ldy,
-                                       void* stream) {
-  if (count < 1 || count > FAIRY2I_MAX_GROUP || !codes || !scales || !y)
+fairy2i_status fairy2i_wl_matmul_group_path(const void* x, fairy2i_dtype xdt, int64_t B,
+                                            int64_t in_features, int64_t ldx, int count,
+                                            const uint32_t* const* codes,
+                                            const float* const* scales, int64_t out_features,
+                                            int T, float* const* y, int64_t ldy, int path,
+                                            void* stream) {
+  if (count < 1 || count > FAIRY2I_MAX_GROUP || !codes || !scales || !y ||
+      (path != 0 && path != 1 && path != 4))
     return FAIRY2I_ERR_INVALID_ARG;
   // Every member is validated as a single call would be (B = 0 included) before anything runs.
   for (int g = 0; g < count; ++g) {
@@ -183,7 +215,15 @@ fairy2i_status fairy2i_wl_matmul_group(const void* x, fairy2i_dtype xdt, int64_t
   const int64_t wpr = fairy2i_codes_words_per_row(m);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   bool handled = false;
-  if (B <= 2) {   // one launch of the decode kernel for the whole group
+  if (B <= 2 && (path == 4 || (path == 0 && xdt == FAIRY2I_BF16 && prefer_stream(n, count)))) {
+    // one launch of the persistent tcgen05 decode kernel
+    const fairy2i_status st = launch_wl_stream_group(x, xdt, B, in_features, ldx, count, codes,
+                                                     scales, n, m, out_features, wpr, T, y, ldy,
+                                                     s, &handled);
+    if (handled || st != FAIRY2I_OK) return st;
+    if (path == 4) return FAIRY2I_ERR_INVALID_ARG;
+  }
+  if (B <= 2) {   // one launch of the warp-MMA decode kernel for the whole group
     const fairy2i_status st = launch_wl_decode_group(x, xdt, B, in_features, ldx, count, codes,
                                                      scales, n, m, out_features, wpr, T, y, ldy,
                                                      s, &handled);
@@ -196,6 +236,15 @@ fairy2i_status fairy2i_wl_matmul_group(const void* x, fairy2i_dtype xdt, int64_t
     if (st != FAIRY2I_OK) return st;
   }
   return FAIRY2I_OK;
+}
+
+fairy2i_status fairy2i_wl_matmul_group(const void* x, fairy2i_dtype xdt, int64_t B,
+                                       int64_t in_features, int64_t ldx, int count,
+                                       const uint32_t* const* codes, const float* const* scales,
+                                       int64_t out_features, int T, float* const* y, int64_t ldy,
+                                       void* stream) {
+  return fairy2i_wl_matmul_group_path(x, xdt, B, in_features, ldx, count, codes, scales,
+                                      out_features, T, y, ldy, 0, stream);
 }
 
 fairy2i_status fairy2i_codes_adjoint(const uint32_t* codes, int64_t n, int64_t m, int T,

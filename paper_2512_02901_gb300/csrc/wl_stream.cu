@@ -1,0 +1,832 @@
+// Persistent decode (B <= 2 tokens) kernel of the quantized widely-linear matmul on the
+// 5th-generation tensor cores: the packed codes stream through shared memory, are decoded into
+// tensor memory and multiplied there (tcgen05.mma, kind::f8f6f4, A in TMEM).
+//
+// Arithmetic (Eq. ifairy-dequant, Algorithm 1 with the W conj(x) term). Every code carries the
+// signs sigma = sign(Re b + Im b), tau = sign(Re b - Im b) of its codeword b; with
+// h = (s_re + i s_im)/2 the dequantized weight is h sigma + conj(h) tau. Per (stage t, matrix)
+// a row needs P = sum_k sigma_k x_k and Q = sum_k tau_k x_k; then y += h P + conj(h) Q for U and
+// h conj(P) + conj(h) conj(Q) for W (the conj(x) term of Eq. widely-linear).
+//
+// Tensor-core form. TMEM lane L = tm R + r holds row r of stage-matrix tm = 2 t + matrix
+// (R = 64, 32, 16, 16 rows for T = 1..4). One MMA (M = 128, N = 16, K = 32, e4m3 x e4m3 -> f32)
+// covers one code word (16 codes) of the 128 lanes. A word becomes 32 A bytes, (sigma_2j,
+// sigma_2j+1, tau_2j, tau_2j+1) for j = 0..7, each an e4m3 value affine in its bit by one LOP3
+// per four bytes (a = alpha + 2 bit, sigma = (1 + alpha) - a), so P = C - D, D the MMA result
+// and C = sum_k (1 + alpha_k) x_k the same for every row. B holds x split exactly into two e4m3
+// limbs (hi = e4m3(x S), lo = e4m3(64 (x S - hi)), S a power of two per CTA and token) in the
+// 16 columns (token, limb, sigma/tau slot, re/im).
+//
+// Work. A job is one row block (R rows of every stage-matrix) of one linear of the group; the
+// jobs are dealt round-robin to thread-block clusters of ks CTAs, and rank r of a cluster takes
+// the 128-code chunks [r nch / ks, (r+1) nch / ks) of every job, so a CTA's K range (and its
+// x-dependent operands: the B tiles, C and S) is the same for all its jobs and is built once per
+// launch. A unit is one chunk of one job (4 KB of codes: one 512-byte block per 16-row tile of
+// every stage-matrix); a stage of the shared-memory ring holds one job's units, which arrive as
+// one bulk copy per tile (the chunks of a tile are adjacent in memory). The grid holds at most
+// one wave of resident clusters, so every CTA loops over its jobs and the launch has no tail
+// wave. Partial rows are summed in distributed shared memory in rank order (deterministic);
+// rank 0 writes y.
+//
+// Programmatic dependent launch. Only x (and y) may belong to the previous kernel in the stream:
+// the copies of the codes into the shared-memory ring and their decoding into tensor memory
+// start before griddepcontrol.wait; the B tiles, and with them every MMA, come after it.
+//
+// Roles (17 warps): warps 0-7 are two decoder sets of four (warp w reaches TMEM lanes
+// 32 (w % 4) ..), set s decoding units q = s, s + 2, ... into its three A slots; warp 8 streams
+// the codes; lane 0 of warp 9 + 2 s + e issues the MMAs of words 4e .. 4e + 3 of every unit of
+// set s into its own accumulator of the job's buffer (two buffers, so a job's read-out overlaps
+// the next job's MMAs); warps 13-16 load x, build the B tiles, C and S, then read out, combine
+// and reduce every job's accumulators and write y.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_fp8.h>
+
+#include <mutex>
+
+#include "common.cuh"
+#include "ptx.cuh"
+#include "tc.cuh"
+
+namespace fairy2i {
+
+namespace sd {
+
+constexpr int kSets = 2;                      // decoder sets of four warps
+constexpr int kSlots = 3;                     // A slots per set (one unit, 64 TMEM columns)
+constexpr int kIss = 2;                       // MMA-issuing threads per set (words 0-3, 4-7)
+constexpr int kDecWarps = 4 * kSets;          // warps 0-7
+constexpr int kCopyWarp = kDecWarps;          // 8
+constexpr int kIssWarp0 = kCopyWarp + 1;      // 9-12: warp kIssWarp0 + kIss s + e
+constexpr int kEpiWarp0 = kIssWarp0 + kSets * kIss;   // 13-16 (warp % 4 = 1, 2, 3, 0)
+constexpr int kWarps = kEpiWarp0 + 4;         // 17
+constexpr int kThreads = kWarps * 32;         // 544
+constexpr int kEpiThreads = 128;
+constexpr int kRingBytes = 112 * 1024;        // code ring: one job (nu units) per stage
+constexpr int kMaxStages = 14;
+constexpr int kUnitBytes = 4096;              // codes of one unit (8 tiles x 512 B)
+constexpr int kWordB = 528;                   // B tile of one word: 16 rows x 32 bytes, + 16 B
+                                              // so that the tiles of consecutive words start in
+                                              // different shared-memory banks
+constexpr int kChunkB = 8 * kWordB;           // B tiles of one chunk
+constexpr int kMaxU = 12;                     // chunks per CTA
+constexpr int kMaxCluster = 8;
+constexpr int kMaxGroup = 4;
+constexpr int kPart = 256;                    // floats of one partial (R rows x NB x 2)
+constexpr int kAccCols = 16;
+constexpr int kNumAcc = kSets * kIss;         // accumulators per job buffer
+constexpr int kColSlots = 2 * kNumAcc * kAccCols;   // accumulators: [buffer][set][issuer] x 16
+constexpr int kTmemCols = 512;
+constexpr uint64_t kWaitNs = 1000000000ull;   // 1 s: a pipeline wait is microseconds
+constexpr uint32_t kIdesc = idesc_e4m3_f32(128, 16);
+static_assert(kColSlots + kSets * kSlots * 64 <= kTmemCols, "TMEM columns");
+
+// Shared memory layout (bytes from the 1024-aligned base).
+constexpr int kOffRing = 0;
+constexpr int kOffB = kOffRing + kRingBytes;                      // 112 KB
+constexpr int kOffRed = kOffB + kMaxU * kChunkB;                  // + 50 KB
+constexpr int kOffGather = kOffRed + 128 * 2 * 2 * 4;             // + 2 KB
+constexpr int kOffBar = kOffGather + 2 * kMaxCluster * kPart * 4; // + 16 KB
+constexpr int kNumBars = 2 * kMaxStages + 2 * kSets * kSlots + 2 + 2 + 1 + 2 + 2 + kNumAcc;
+constexpr int kOffMisc = kOffBar + kNumBars * 8;
+constexpr int kSmemBytes = kOffMisc + 512 + 1024;                 // + alignment slack
+// One CTA per SM: it owns all TMEM columns (a second CTA on the SM would wait in its allocation),
+// and no two CTAs of a launch share an SM's tensor core.
+static_assert(kSmemBytes > 116 * 1024, "one CTA per SM");
+static_assert(kSmemBytes <= 227 * 1024, "shared memory per CTA");
+
+struct Args {
+  const uint32_t* codes[kMaxGroup];
+  const float* scales[kMaxGroup];
+  float* y[kMaxGroup];
+  const __nv_bfloat16* x;
+  unsigned int* status;
+  int64_t B, in_features, ldx, n, m, out_features, ldy;
+  int G;          // linears in the group
+  int nch;        // 128-code chunks per row
+  int row_tiles;  // ceil(n / 16)
+  int rbs;        // row blocks per linear, ceil(n / R)
+  int ks;         // CTAs per cluster
+  int nclusters;  // clusters in the grid
+  int x_vec;      // x rows 16-byte aligned with m % 8 == 0: vector loads allowed
+  int x_bulk;     // and in_features even: the x slice is prefetched to L2 in one range
+};
+
+struct Misc {
+  uint32_t tmem;
+  int abort;
+  unsigned int xmax[4][2];       // per epilogue warp and token: max |x| as float bits
+  float scl[kMaxGroup][16];      // scales of the group: [linear][(stage, matrix, re/im)]
+  float cpart[4][4];             // per epilogue warp: [token][part] partial C
+};
+
+__device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort,
+                                              unsigned int* status) {
+  if (*abort) return false;
+  if (mbar_wait_timed(bar, parity, kWaitNs)) return true;
+  *abort = 1;
+  latch_status(status, kStatusTimeout);
+  return false;
+}
+
+// A register j (0..7) of a word: e4m3 bytes (sigma_2j, sigma_2j+1, tau_2j, tau_2j+1), each
+// alpha_q + 2 bit with q the bit position used (2, 3, 2, 3, 6, 7, 6, 7 for j = 0..7; the word
+// shifted left by 2 for j in {0, 1, 4, 5}); 1 + alpha = 5, 3, 5, 3, 1, 0, 1, 0.
+__device__ __forceinline__ void decode_word(uint32_t w0, uint32_t* r) {
+  const uint32_t w2 = w0 << 2;
+  r[0] = lop3_and_or(w2, 0x04040404u, 0x48484848u);   // q = 2: 4 + 2 bit
+  r[1] = lop3_and_or(w2, 0x08080808u, 0x40404040u);   // q = 3: 2 + 2 bit
+  r[2] = lop3_and_or(w0, 0x04040404u, 0x48484848u);
+  r[3] = lop3_and_or(w0, 0x08080808u, 0x40404040u);
+  r[4] = w2 & 0x40404040u;                            // q = 6: 0 + 2 bit
+  r[5] = lop3_and_xor(w2, 0x80808080u, 0xB8B8B8B8u);  // q = 7: -1 + 2 bit
+  r[6] = w0 & 0x40404040u;
+  r[7] = lop3_and_xor(w0, 0x80808080u, 0xB8B8B8B8u);
+}
+
+__device__ __forceinline__ float bf_lo(uint32_t v) { return __uint_as_float(v << 16); }
+__device__ __forceinline__ float bf_hi(uint32_t v) { return __uint_as_float(v & 0xffff0000u); }
+
+__device__ __forceinline__ uint32_t e4m3x2(float a, float b) {
+  return (uint32_t)__nv_cvt_float2_to_fp8x2(make_float2(a, b), __NV_SATFINITE, __NV_E4M3);
+}
+__device__ __forceinline__ float2 e4m3x2_to_float2(uint32_t v) {
+  return __half22float2(
+      __half2(__nv_cvt_fp8x2_to_halfraw2((__nv_fp8x2_storage_t)v, __NV_E4M3)));
+}
+
+// Power-of-two S with max|x| S < 128, and 1/S, from the exponent bits of max|x|.
+__device__ __forceinline__ void pow2_scale(float mx, float& S, float& invS) {
+  const int E = (int)((__float_as_uint(mx) >> 23) & 0xffu);
+  if (E >= 7 && E <= 254) {
+    S = __uint_as_float((uint32_t)(260 - E) << 23);
+    invS = __uint_as_float((uint32_t)(E - 6) << 23);
+  } else {
+    S = 1.f;
+    invS = 1.f;
+  }
+}
+
+// Eight bf16 values of part `part` of token b at complex index k (k % 8 == 0), zero outside
+// the valid range of that part. Plain (coherent) loads: x may come from the previous kernel.
+__device__ __forceinline__ uint4 load_x8(const Args& a, int b, int part, int64_t k) {
+  const __nv_bfloat16* row = a.x + (int64_t)b * a.ldx + (int64_t)part * a.m;
+  const int64_t lim = part ? a.in_features - a.m : a.m;
+  if (a.x_vec && k + 8 <= lim) return *reinterpret_cast<const uint4*>(row + k);
+  uint32_t w[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int64_t k0 = k + 2 * i, k1 = k0 + 1;
+    const uint32_t lo = k0 < lim ? (uint32_t)__bfloat16_as_ushort(row[k0]) : 0u;
+    const uint32_t hi = k1 < lim ? (uint32_t)__bfloat16_as_ushort(row[k1]) : 0u;
+    w[i] = lo | (hi << 16);
+  }
+  return make_uint4(w[0], w[1], w[2], w[3]);
+}
+
+// Job index i of this cluster -> (linear g, row block rb).
+__device__ __forceinline__ void job_of(const Args& a, int cluster, int i, int& g, int& rb) {
+  const int J = cluster + i * a.nclusters;
+  g = J / a.rbs;
+  rb = J - g * a.rbs;
+}
+
+template <int NB, int T>
+__global__ void __launch_bounds__(kThreads, 1) wl_stream_kernel(const Args a) {
+  constexpr int TM = 2 * T;
+  constexpr int R = (T == 1) ? 64 : (T == 2 ? 32 : 16);  // rows per row block
+  constexpr int RT = R / 16;                              // 16-row code tiles per row block
+  constexpr int NV = R * NB * 2;                          // outputs of a row block
+  static_assert(TM * RT * 512 <= kUnitBytes, "unit size");
+  static_assert(NV <= kPart && NV <= 2 * kEpiThreads, "partial size");
+  extern __shared__ unsigned char smem_raw[];
+  unsigned char* smem = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kOffBar);
+  uint64_t* full = bars;                        // [stage] codes landed        (tx count)
+  uint64_t* empty = full + kMaxStages;          // [stage] codes read          (4 warps x nu)
+  uint64_t* sfull = empty + kMaxStages;         // [set][slot] A written       (4 warps)
+  uint64_t* sfree = sfull + kSets * kSlots;     // [set][slot] its MMAs done   (kIss commits)
+  uint64_t* jfull = sfree + kSets * kSlots;     // [buffer] job accumulated    (kNumAcc issuers)
+  uint64_t* jfree = jfull + 2;                  // [buffer] job read out       (4 warps)
+  uint64_t* bready = jfree + 2;                 // B tiles written             (1 arrival)
+  uint64_t* gfull = bready + 1;                 // [buffer] rank 0: partials arrived
+  uint64_t* gfree = gfull + 2;                  // [buffer] ranks > 0: rank 0 read the buffer
+  uint64_t* fin = gfree + 2;                    // [issuer] abort path
+  Misc* misc = reinterpret_cast<Misc*>(smem + kOffMisc);
+  volatile int* abort_flag = &misc->abort;
+  float* red = reinterpret_cast<float*>(smem + kOffRed);
+  float* gather = reinterpret_cast<float*>(smem + kOffGather);          // [buf][rank][kPart]
+
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int ks = a.ks;
+  const int rank = ks > 1 ? (int)cluster_ctarank() : 0;
+  const int cluster = (int)(blockIdx.x / (unsigned)ks);
+  const int c0 = (rank * a.nch) / ks;
+  const int nu = ((rank + 1) * a.nch) / ks - c0;          // units per job (>= 1)
+  const int njobs_all = a.G * a.rbs;
+  const int njobs = cluster < njobs_all ? (njobs_all - 1 - cluster) / a.nclusters + 1 : 0;
+  const int total = njobs * nu;                           // units of this CTA
+  const int stage_bytes = nu * kUnitBytes;                // one job: [tile][unit][512 B]
+  const int nstages = min(kMaxStages, kRingBytes / stage_bytes);
+
+  // ---- prologue: barriers (the lanes of warp 1), TMEM (warp 0) ----
+  if (warp == 1) {
+    for (int i = lane; i < kNumBars; i += 32) {
+      uint32_t cnt = 1;
+      if (i >= kMaxStages && i < 2 * kMaxStages) cnt = 4 * nu;                         // empty
+      else if (i >= 2 * kMaxStages && i < 2 * kMaxStages + kSets * kSlots) cnt = 4;    // sfull
+      else if (i < 2 * kMaxStages + 2 * kSets * kSlots && i >= 2 * kMaxStages) cnt = kIss;
+      else if (bars + i == jfull || bars + i == jfull + 1) cnt = kNumAcc;
+      else if (bars + i == jfree || bars + i == jfree + 1) cnt = 4;
+      else if (bars + i == gfull || bars + i == gfull + 1) cnt = ks > 1 ? (ks - 1) * kEpiThreads : 1;
+      mbar_init(bars + i, cnt);
+    }
+    if (lane == 0) misc->abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0) tmem_alloc(&misc->tmem, kTmemCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (ks > 1) cluster_arrive();   // barriers of every rank initialised (waited before DSMEM use)
+  const uint32_t tmem = misc->tmem;
+  pdl_launch_dependents();
+
+  if (warp < kDecWarps) {
+    // ---------------- decoder sets: one unit into one A slot at a time ----------------
+    const int set = warp >> 2, quarter = warp & 3;
+    const int L = quarter * 32 + lane;                       // TMEM lane of this thread
+    const int tm = L / R, r = L % R;
+    // this lane's 8 words of unit u inside a stage: tile tm RT + r / 16, row r % 16 (32 bytes)
+    const uint32_t lane_off = (uint32_t)((tm * RT + r / 16) * nu * 512 + (r % 16) * 32);
+    const uint32_t ring = smem_u32(smem + kOffRing);
+    const uint32_t t_lane = tmem + ((uint32_t)(quarter * 32) << 16) + kColSlots;
+    int l = 0;
+    for (int q = set; q < total; q += kSets, ++l) {
+      const int i = q / nu, u = q - i * nu;
+      const int st = i % nstages, sl = l % kSlots, si = set * kSlots + sl;
+      if (!__all_sync(0xffffffffu, wait_or_abort(&full[st], (i / nstages) & 1, abort_flag,
+                                                  a.status)))
+        break;
+      const uint32_t src = ring + st * stage_bytes + lane_off + u * 512;
+      const uint4 q0 = lds128(src), q1 = lds128(src + 16);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty[st]);
+      // Units past the first kSlots need MMAs, i.e. x: wait for the previous kernel first, so
+      // that no bounded wait below counts its run time.
+      if (l == kSlots) pdl_wait_primary();
+      if (l >= kSlots &&   // the slot's previous unit has been multiplied
+          !__all_sync(0xffffffffu, wait_or_abort(&sfree[si], ((l / kSlots) - 1) & 1, abort_flag,
+                                                  a.status)))
+        break;
+      const uint32_t a_col = t_lane + si * 64;
+      uint32_t rr[32];
+      decode_word(q0.x, rr);
+      decode_word(q0.y, rr + 8);
+      decode_word(q0.z, rr + 16);
+      decode_word(q0.w, rr + 24);
+      tmem_st32(a_col, rr);
+      decode_word(q1.x, rr);
+      decode_word(q1.y, rr + 8);
+      decode_word(q1.z, rr + 16);
+      decode_word(q1.w, rr + 24);
+      tmem_st32(a_col + 32, rr);
+      tmem_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sfull[si]);
+    }
+  } else if (warp == kCopyWarp) {
+    // ---------------- code stream: one stage per job, one bulk copy per tile ----------------
+    const int tmi = lane / RT, rt = lane % RT;
+    int issued = 0;
+    for (int i = 0; i < njobs; ++i) {
+      const int st = i % nstages;
+      if (i == nstages) pdl_wait_primary();   // refills wait on MMAs, i.e. on x
+      if (i >= nstages) {
+        const bool ok = lane != 0 || wait_or_abort(&empty[st], ((i / nstages) - 1) & 1,
+                                                   abort_flag, a.status);
+        if (!__all_sync(0xffffffffu, ok)) break;
+      }
+      int g, rb;
+      job_of(a, cluster, i, g, rb);
+      int nrt = 0;   // existing 16-row tiles of the row block
+#pragma unroll
+      for (int k = 0; k < RT; ++k) nrt += (rb * RT + k < a.row_tiles) ? 1 : 0;
+      if (lane == 0) mbar_arrive_expect_tx(&full[st], (uint32_t)(TM * nrt * nu * 512));
+      __syncwarp();
+      if (lane < TM * RT && rt < nrt) {
+        const int64_t tile = (int64_t)tmi * a.row_tiles + rb * RT + rt;
+        bulk_load(smem + kOffRing + st * stage_bytes + lane * nu * 512,
+                  a.codes[g] + (tile * a.nch + c0) * 128, (uint32_t)(nu * 512), &full[st]);
+      }
+      issued = i + 1;
+    }
+    // Abort path: every issued copy lands before shared memory is released.
+    if (lane == 0 && *abort_flag) {
+      for (int i = (issued > nstages ? issued - nstages : 0); i < issued; ++i)
+        (void)mbar_wait_timed(&full[i % nstages], (i / nstages) & 1, 1000000ull);
+    }
+  } else if (warp < kEpiWarp0) {
+    // ------ MMA issuers: lane 0 of warp kIssWarp0 + kIss s + e issues words 4e .. 4e+3 of every
+    // unit of set s into its own accumulator of the job's buffer ------
+    const int ii = warp - kIssWarp0, set = ii / kIss, e = ii % kIss;
+    if (lane == 0) {
+      const uint32_t b_base = smem_u32(smem + kOffB);
+      pdl_wait_primary();   // the B tiles are built from x after the previous kernel
+      bool ok = wait_or_abort(bready, 0, abort_flag, a.status);
+      tc_fence_after();
+      bool issued = false;
+      int l = 0, cur = -1;
+      bool first = true;
+      // Before touching job i's accumulator buffer, the read-out of job i - 2 must be done; a
+      // job without a unit of this set still gets this issuer's arrival.
+      auto enter_job = [&](int i) {
+        if (i >= 2 && ok) ok = wait_or_abort(&jfree[i & 1], ((i >> 1) - 1) & 1, abort_flag, a.status);
+      };
+      for (int q = set; ok && q < total; q += kSets, ++l) {
+        const int i = q / nu, u = q - i * nu;
+        if (i != cur) {
+          if (cur >= 0) mma_commit(&jfull[cur & 1]);
+          for (int i2 = cur + 1; ok && i2 < i; ++i2) {   // jobs without a unit of this set
+            enter_job(i2);
+            if (ok) mbar_arrive(&jfull[i2 & 1]);
+          }
+          enter_job(i);
+          if (!ok) break;
+          tc_fence_after();
+          cur = i;
+          first = true;
+        }
+        const int si = set * kSlots + l % kSlots;
+        ok = wait_or_abort(&sfull[si], (l / kSlots) & 1, abort_flag, a.status);
+        if (!ok) break;
+        tc_fence_after();
+        const uint32_t a_slot = tmem + kColSlots + si * 64;
+        const uint32_t d_tmem = tmem + ((cur & 1) * kNumAcc + ii) * kAccCols;
+        const uint32_t bt = b_base + u * kChunkB;
+#pragma unroll
+        for (int w4 = 0; w4 < 4; ++w4) {
+          const int w = e * 4 + w4;
+          mma_e4m3_ts(d_tmem, a_slot + w * 8, smem_desc(bt + w * kWordB, 128, 256), kIdesc,
+                      (first && w4 == 0) ? 0u : 1u);
+        }
+        first = false;
+        issued = true;
+        mma_commit(&sfree[si]);
+      }
+      if (ok) {
+        if (cur >= 0) mma_commit(&jfull[cur & 1]);
+        for (int i2 = cur + 1; ok && i2 < njobs; ++i2) {
+          enter_job(i2);
+          if (ok) mbar_arrive(&jfull[i2 & 1]);
+        }
+      }
+      // Abort path: the MMAs this thread issued finish before TMEM is released.
+      if (issued && *abort_flag) {
+        mma_commit(&fin[ii]);
+        (void)mbar_wait_timed(&fin[ii], 0, kWaitNs);
+      }
+    }
+    __syncwarp();
+  } else {
+    // ---------------- x -> B tiles, C, S; then the read-out of every job ----------------
+    const int et = tid - kEpiWarp0 * 32;        // 0 .. 127
+    const int ew = warp - kEpiWarp0;            // 0 .. 3
+    const int quarter = warp & 3;
+    const int L = quarter * 32 + lane;
+    const int64_t kbeg = (int64_t)c0 * 128;
+    // Before the wait: zero the B tiles (rows of unused tokens stay zero) and warm L2 with the
+    // x slice.
+    for (int o = et; o < nu * kChunkB / 16; o += kEpiThreads)
+      *reinterpret_cast<uint4*>(smem + kOffB + o * 16) = make_uint4(0, 0, 0, 0);
+    // the scales, like the codes, are not written by the previous kernel
+    if (et < a.G * TM * 2) misc->scl[et / (TM * 2)][et % (TM * 2)] = __ldg(a.scales[et / (TM * 2)] + et % (TM * 2));
+    if (a.x_bulk && et < 2 * NB && et / 2 < a.B) {
+      const int b = et >> 1, p = et & 1;
+      const int64_t lim = p ? a.in_features - a.m : a.m;
+      const int64_t k1 = min((int64_t)(c0 + nu) * 128, lim);
+      if (k1 > kbeg)
+        prefetch_l2_bulk(a.x + (int64_t)b * a.ldx + (int64_t)p * a.m + kbeg,
+                         (uint32_t)((k1 - kbeg) * 2));
+    }
+    pdl_wait_primary();               // x may be written by the previous kernel
+    // This thread's groups: for token b and part p, the 8-value groups v = et + 128 jv of the
+    // slice (v < 16 nu), values x_p[8 v .. 8 v + 7].
+    constexpr int kJv = 2;                      // 16 kMaxU / 128 groups per (b, p) and thread
+    static_assert(16 * kMaxU <= kJv * kEpiThreads, "x groups per thread");
+    uint4 xv[NB][2][kJv];
+#pragma unroll
+    for (int b = 0; b < NB; ++b)
+#pragma unroll
+      for (int p = 0; p < 2; ++p)
+#pragma unroll
+        for (int jv = 0; jv < kJv; ++jv) {
+          const int v = et + jv * kEpiThreads;
+          xv[b][p][jv] = (v < nu * 16 && b < a.B) ? load_x8(a, b, p, kbeg + v * 8)
+                                                  : make_uint4(0, 0, 0, 0);
+        }
+    // max |x| per token (non-negative float bits order like unsigned integers)
+#pragma unroll
+    for (int b = 0; b < NB; ++b) {
+      unsigned int mx = 0u;
+#pragma unroll
+      for (int p = 0; p < 2; ++p)
+#pragma unroll
+        for (int jv = 0; jv < kJv; ++jv) {
+          const uint32_t ev[4] = {xv[b][p][jv].x, xv[b][p][jv].y, xv[b][p][jv].z, xv[b][p][jv].w};
+#pragma unroll
+          for (int i = 0; i < 4; ++i) mx = max(mx, max((ev[i] << 17) >> 1, ev[i] & 0x7fff0000u));
+        }
+      mx = __reduce_max_sync(0xffffffffu, mx);
+      if (lane == 0) misc->xmax[ew][b] = mx;
+    }
+    named_bar_sync(1, kEpiThreads);
+    float S[2] = {1.f, 1.f}, invS[2] = {1.f, 1.f};
+#pragma unroll
+    for (int b = 0; b < NB; ++b) {
+      const unsigned int xm = max(max(misc->xmax[0][b], misc->xmax[1][b]),
+                                  max(misc->xmax[2][b], misc->xmax[3][b]));
+      pow2_scale(__uint_as_float(xm), S[b], invS[b]);
+    }
+    // B tiles and C. Group v = 16 u + 2 w + hh of token b, part p: the values x_p[k], k = 128 u +
+    // 16 w + 8 hh .. + 7, become the 16-byte halves hh of the four rows (limb, slot, p) of token b
+    // in the tile of word w of chunk u: register j' (codes 2j, 2j + 1, j = 4 hh + j') holds the
+    // limb bytes of x[2j], x[2j + 1] in its sigma half (bytes 0-1) or tau half (bytes 2-3).
+    float cacc[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
+#pragma unroll
+    for (int b = 0; b < NB; ++b)
+#pragma unroll
+      for (int p = 0; p < 2; ++p)
+#pragma unroll
+        for (int jv = 0; jv < kJv; ++jv) {
+          const int v = et + jv * kEpiThreads;
+          if (v < nu * 16) {
+            const int u = v >> 4, w = (v >> 1) & 7, hh = v & 1;
+            const uint32_t ev[4] = {xv[b][p][jv].x, xv[b][p][jv].y, xv[b][p][jv].z,
+                                    xv[b][p][jv].w};
+            uint32_t hp[4], lp[4];   // limb byte pairs (x[2j], x[2j+1]) of register j'
+            float cs = 0.f;
+#pragma unroll
+            for (int jj = 0; jj < 4; ++jj) {
+              const float f0 = bf_lo(ev[jj]), f1 = bf_hi(ev[jj]);
+              const float v0 = f0 * S[b], v1 = f1 * S[b];
+              hp[jj] = e4m3x2(v0, v1) & 0xffffu;
+              const float2 hf = e4m3x2_to_float2(hp[jj]);
+              lp[jj] = e4m3x2(64.f * (v0 - hf.x), 64.f * (v1 - hf.y)) & 0xffffu;
+              // 1 + alpha of codes 2j, 2j+1: 5, 3, 5, 3 (first half of a word), 1, 0, 1, 0
+              const float wgt = hh ? ((jj & 1) ? 0.f : 1.f) : ((jj & 1) ? 3.f : 5.f);
+              cs = fmaf(wgt, f0 + f1, cs);
+            }
+            cacc[b][p] += cs;
+            unsigned char* tile = smem + kOffB + u * kChunkB + w * kWordB;
+#pragma unroll
+            for (int limb = 0; limb < 2; ++limb) {
+              const uint32_t* src = limb ? lp : hp;
+#pragma unroll
+              for (int slot = 0; slot < 2; ++slot) {
+                const int nrow = ((b * 2 + limb) * 2 + slot) * 2 + p;
+                const int sh = slot ? 16 : 0;
+                *reinterpret_cast<uint4*>(tile + (nrow >> 3) * 256 + hh * 128 + (nrow & 7) * 16) =
+                    make_uint4(src[0] << sh, src[1] << sh, src[2] << sh, src[3] << sh);
+              }
+            }
+          }
+        }
+    fence_proxy_async_smem();   // generic-proxy writes of B visible to the tensor cores
+    named_bar_sync(1, kEpiThreads);
+    if (et == 0) mbar_arrive(bready);
+#pragma unroll
+    for (int b = 0; b < 2; ++b)
+#pragma unroll
+      for (int p = 0; p < 2; ++p) {
+        float v = cacc[b][p];
+#pragma unroll
+        for (int h = 16; h >= 1; h >>= 1) v += __shfl_xor_sync(0xffffffffu, v, h);
+        if (lane == 0) misc->cpart[ew][b * 2 + p] = v;
+      }
+    named_bar_sync(1, kEpiThreads);
+    float C[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      C[j] = (misc->cpart[0][j] + misc->cpart[1][j]) + (misc->cpart[2][j] + misc->cpart[3][j]);
+
+    // ---- per job: read out, combine with the scales, sum the stage-matrices, reduce ----
+    if (ks > 1) cluster_wait();   // every rank's barriers are initialised
+    const int tmL = L / R;
+    for (int i = 0; i < njobs; ++i) {
+      const int buf = i & 1;
+      int g, rb;
+      job_of(a, cluster, i, g, rb);
+      float d[16];
+#pragma unroll
+      for (int k = 0; k < 16; ++k) d[k] = 0.f;
+      const bool got = __all_sync(0xffffffffu,
+                                  wait_or_abort(&jfull[buf], (i >> 1) & 1, abort_flag, a.status));
+      tc_fence_after();
+      if (got) {
+#pragma unroll
+        for (int s = 0; s < kSets; ++s) {
+          // sets with at least one unit in job i
+          const bool has = nu >= kSets || ((s - i * nu) % kSets + kSets) % kSets < nu;
+          if (has) {
+            float v0[16], v1[16];
+            const uint32_t acc = tmem + ((uint32_t)(quarter * 32) << 16) +
+                                 (buf * kNumAcc + s * kIss) * kAccCols;
+            tmem_ld16(acc, v0);
+            tmem_ld16(acc + kAccCols, v1);
+            tmem_wait_ld();
+#pragma unroll
+            for (int k = 0; k < 16; ++k) d[k] += v0[k] + v1[k];
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&jfree[buf]);
+      if (L < TM * R) {
+        const int t = tmL >> 1;
+        const bool mat = tmL & 1;
+        const float hr = 0.5f * misc->scl[g][(t * 2 + mat) * 2 + 0];
+        const float hi = 0.5f * misc->scl[g][(t * 2 + mat) * 2 + 1];
+#pragma unroll
+        for (int b = 0; b < NB; ++b) {
+          const float cre = C[b * 2 + 0], cim = C[b * 2 + 1];
+          const float is = invS[b];
+          // column (token, limb, slot, part) = ((b 2 + limb) 2 + slot) 2 + part
+          const int c = b * 8;
+          const float pre = cre - (d[c + 0] + 0.015625f * d[c + 4]) * is;
+          float pim = cim - (d[c + 1] + 0.015625f * d[c + 5]) * is;
+          const float qre = cre - (d[c + 2] + 0.015625f * d[c + 6]) * is;
+          float qim = cim - (d[c + 3] + 0.015625f * d[c + 7]) * is;
+          if (mat) {   // W multiplies conj(x): conjugate P and Q
+            pim = -pim;
+            qim = -qim;
+          }
+          red[(L * NB + b) * 2 + 0] = hr * pre - hi * pim + hr * qre + hi * qim;
+          red[(L * NB + b) * 2 + 1] = hr * pim + hi * pre + hr * qim - hi * qre;
+        }
+      }
+      named_bar_sync(1, kEpiThreads);
+      // Sum over the stage-matrices: value idx = (row rr, token b, re/im).
+      float vals[2];
+#pragma unroll
+      for (int it = 0; it < 2; ++it) {
+        const int idx = et + it * kEpiThreads;
+        float sum = 0.f;
+        if (idx < NV) {
+          const int rr = idx / (NB * 2), rest = idx % (NB * 2);
+#pragma unroll
+          for (int m2 = 0; m2 < TM; ++m2) sum += red[(m2 * R + rr) * NB * 2 + rest];
+        }
+        vals[it] = sum;
+      }
+      named_bar_sync(1, kEpiThreads);   // red is free for the next job
+      bool write = rank == 0;
+      if (ks > 1) {
+        if (rank != 0) {
+          // the buffer of job i - 2 in rank 0 has been read
+          const bool fr = i < 2 || __all_sync(0xffffffffu, wait_or_abort(&gfree[buf], ((i >> 1) - 1) & 1,
+                                                                        abort_flag, a.status));
+          if (fr && !*abort_flag) {
+            const uint32_t g0 = smem_u32(gather) + (uint32_t)((buf * kMaxCluster + rank) * kPart) * 4;
+#pragma unroll
+            for (int it = 0; it < 2; ++it) {
+              const int idx = et + it * kEpiThreads;
+              if (idx < NV) st_cluster_f32(mapa_shared(g0 + idx * 4, 0), vals[it]);
+            }
+          }
+          // arrive even after an abort, so that rank 0 does not wait for the full second
+          mbar_arrive_remote(mapa_shared(smem_u32(&gfull[buf]), 0));
+        } else {
+          // Waited even after an abort: every rank arrives once per job, and rank 0 stays alive
+          // until those remote arrivals (and the partials before them) have landed.
+          const bool got2 = __all_sync(0xffffffffu,
+                                       mbar_wait_cluster_timed(&gfull[buf], (i >> 1) & 1, kWaitNs)) &&
+                            !*abort_flag;
+          if (!got2) {
+            if (!*abort_flag) {
+              *abort_flag = 1;
+              latch_status(a.status, kStatusTimeout);
+            }
+            write = false;
+          } else {
+#pragma unroll
+            for (int it = 0; it < 2; ++it) {
+              const int idx = et + it * kEpiThreads;
+              if (idx < NV)
+                for (int r2 = 1; r2 < ks; ++r2) vals[it] += gather[(buf * kMaxCluster + r2) * kPart + idx];
+            }
+          }
+          named_bar_sync(1, kEpiThreads);   // every read of gather[buf] is done
+          // Rank r waits for this release only before job i + 2; the last two jobs send none, so
+          // no remote access ever reaches a CTA that has passed its last wait.
+          if (et < ks - 1 && i + 2 < njobs)
+            mbar_arrive_remote(mapa_shared(smem_u32(&gfree[buf]), et + 1));
+        }
+      }
+      if (write && !*abort_flag) {
+#pragma unroll
+        for (int it = 0; it < 2; ++it) {
+          const int idx = et + it * kEpiThreads;
+          if (idx < NV) {
+            const int rr = idx / (NB * 2), b = (idx >> 1) % NB, comp = idx & 1;
+            const int64_t jr = (int64_t)rb * R + rr;
+            if (b < a.B && jr < a.n) {
+              float* yb = a.y[g] + (int64_t)b * a.ldy;
+              if (comp == 0) yb[jr] = vals[it];
+              else if (a.n + jr < a.out_features) yb[a.n + jr] = vals[it];
+            }
+          }
+        }
+      }
+    }
+  }
+
+  // Teardown. The first cluster barrier was waited by the epilogue warps; every other thread
+  // waits it here. No second cluster barrier is needed: every remote access targets a CTA that
+  // waits for it (rank 0 for the partials of every job, rank r > 0 for the release of a gather
+  // buffer it writes again).
+  if (ks > 1 && warp < kEpiWarp0) cluster_wait();
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 0) tmem_dealloc(tmem, kTmemCols);
+}
+
+template <int NB, int T>
+fairy2i_status launch(const Args& a, int64_t grid, cudaStream_t stream) {
+  auto kern = wl_stream_kernel<NB, T>;
+  static bool configured = false;
+  if (!configured) {
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) !=
+        cudaSuccess)
+      return FAIRY2I_ERR_CUDA;
+    configured = true;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = (unsigned)a.ks;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  if (cudaLaunchKernelEx(&cfg, kern, a) != cudaSuccess) return FAIRY2I_ERR_CUDA;
+  return FAIRY2I_OK;
+}
+
+// Clusters of `ks` CTAs that can be resident at once on the device (0 if none).
+template <int NB, int T>
+int max_clusters(int ks) {
+  auto kern = wl_stream_kernel<NB, T>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) !=
+      cudaSuccess)
+    return 0;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)(ks * 256));
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = kSmemBytes;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = (unsigned)ks;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return 0;
+  }
+  return n;
+}
+
+}  // namespace sd
+
+namespace {
+std::mutex g_sd_mu;
+int g_sd_clusters[64][4][8][2];   // [device][ks index][T][NB] resident clusters, -1 = unknown
+bool g_sd_init[64];
+}  // namespace
+
+static int sd_resident_clusters(int dev, int ks_idx, int T, int NB) {
+  std::lock_guard<std::mutex> lock(g_sd_mu);
+  if (!g_sd_init[dev]) {
+    for (int i = 0; i < 4; ++i)
+      for (int t = 0; t < 8; ++t)
+        for (int b = 0; b < 2; ++b) g_sd_clusters[dev][i][t][b] = -1;
+    g_sd_init[dev] = true;
+  }
+  int& v = g_sd_clusters[dev][ks_idx][T - 1][NB - 1];
+  if (v < 0) {
+    const int ks = 1 << ks_idx;
+    int r = 0;
+    switch (T * 4 + NB) {
+      case 1 * 4 + 1: r = sd::max_clusters<1, 1>(ks); break;
+      case 1 * 4 + 2: r = sd::max_clusters<2, 1>(ks); break;
+      case 2 * 4 + 1: r = sd::max_clusters<1, 2>(ks); break;
+      case 2 * 4 + 2: r = sd::max_clusters<2, 2>(ks); break;
+      case 3 * 4 + 1: r = sd::max_clusters<1, 3>(ks); break;
+      case 3 * 4 + 2: r = sd::max_clusters<2, 3>(ks); break;
+      case 4 * 4 + 1: r = sd::max_clusters<1, 4>(ks); break;
+      case 4 * 4 + 2: r = sd::max_clusters<2, 4>(ks); break;
+    }
+    v = r;
+  }
+  return v;
+}
+
+// Cluster size and cluster count for `jobs` row blocks of `nch` chunks: ks in {1, 2, 4, 8} with
+// at least one and at most kMaxU chunks per CTA, one wave of resident clusters of at most one CTA
+// per SM, minimising the estimated time jobs-per-cluster x (chunks per CTA + a per-job cost of
+// about a quarter chunk), then the fewest clusters that keep that busiest-cluster load.
+struct SdPlan {
+  int ks = 0, nclusters = 0;
+};
+static SdPlan sd_plan(int dev, int64_t jobs, int64_t nch, int T, int NB) {
+  SdPlan best;
+  int64_t best_cost = -1;
+  int sms = 0;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1)
+    return best;
+  for (int ki = 0; ki < 4; ++ki) {
+    const int ks = 1 << ki;
+    if (nch < ks || (nch + ks - 1) / ks > sd::kMaxU) continue;
+    // one CTA per SM (the kernel's shared memory allows no second one)
+    const int resident = std::min(sd_resident_clusters(dev, ki, T, NB), sms / ks);
+    if (resident < 1) continue;
+    const int64_t per = (jobs + resident - 1) / resident;     // jobs of the busiest cluster
+    // the fewest clusters with that load: the SMs left free start the next kernel early
+    const int64_t nclusters = (jobs + per - 1) / per;
+    const int64_t cost = per * (4 * ((nch + ks - 1) / ks) + 1);   // a job's epilogue ~ 1/4 chunk
+    if (best_cost < 0 || cost < best_cost) {
+      best_cost = cost;
+      best.ks = ks;
+      best.nclusters = (int)nclusters;
+    }
+  }
+  return best;
+}
+
+// `count` linears of the same shape sharing x. Handles B <= 2 bf16 tokens, T <= 4 and rows of at
+// most 8 kMaxU chunks; anything else is left to the other kernels (*handled = false).
+fairy2i_status launch_wl_stream_group(const void* x, fairy2i_dtype xdt, int64_t B,
+                                      int64_t in_features, int64_t ldx, int count,
+                                      const uint32_t* const* codes, const float* const* scales,
+                                      int64_t n, int64_t m, int64_t out_features, int64_t wpr,
+                                      int T, float* const* y, int64_t ldy, cudaStream_t stream,
+                                      bool* handled) {
+  using namespace sd;
+  *handled = false;
+  if (xdt != FAIRY2I_BF16 || B < 1 || B > 2 || T > 4 || count < 1 || count > kMaxGroup)
+    return FAIRY2I_OK;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return FAIRY2I_ERR_CUDA;
+  const int NB = (int)B;
+  const int R = T == 1 ? 64 : (T == 2 ? 32 : 16);
+  const int64_t rbs = (n + R - 1) / R;
+  const int64_t nch = wpr / 8;
+  const int64_t jobs = rbs * count;
+  if (jobs > (int64_t(1) << 30) || nch > (int64_t(1) << 20)) return FAIRY2I_OK;
+  const SdPlan plan = sd_plan(dev, jobs, nch, T, NB);
+  if (plan.ks < 1) return FAIRY2I_OK;
+  Args a;
+  for (int g = 0; g < kMaxGroup; ++g) {
+    a.codes[g] = codes[g < count ? g : 0];
+    a.scales[g] = scales[g < count ? g : 0];
+    a.y[g] = y[g < count ? g : 0];
+  }
+  a.x = reinterpret_cast<const __nv_bfloat16*>(x);
+  a.status = device_status_word();
+  a.B = B; a.in_features = in_features; a.ldx = ldx; a.n = n; a.m = m;
+  a.out_features = out_features; a.ldy = ldy;
+  a.G = count; a.nch = (int)nch; a.row_tiles = (int)((n + 15) / 16); a.rbs = (int)rbs;
+  a.ks = plan.ks; a.nclusters = plan.nclusters;
+  a.x_vec = (reinterpret_cast<uintptr_t>(x) % 16 == 0) && (ldx % 8 == 0) && (m % 8 == 0);
+  a.x_bulk = a.x_vec && (in_features % 2 == 0);
+  const int64_t grid = (int64_t)plan.nclusters * plan.ks;
+  *handled = true;
+  switch (T * 4 + NB) {
+    case 1 * 4 + 1: return launch<1, 1>(a, grid, stream);
+    case 1 * 4 + 2: return launch<2, 1>(a, grid, stream);
+    case 2 * 4 + 1: return launch<1, 2>(a, grid, stream);
+    case 2 * 4 + 2: return launch<2, 2>(a, grid, stream);
+    case 3 * 4 + 1: return launch<1, 3>(a, grid, stream);
+    case 3 * 4 + 2: return launch<2, 3>(a, grid, stream);
+    case 4 * 4 + 1: return launch<1, 4>(a, grid, stream);
+    case 4 * 4 + 2: return launch<2, 4>(a, grid, stream);
+  }
+  *handled = false;
+  return FAIRY2I_OK;
+}
+
+}  // namespace fairy2i

@@ -89,7 +89,7 @@ def test_wl_matmul_validation(lib):
         return lib.fairy2i_wl_matmul_path(x, xdt, B, inf, ldx, codes, scales, outf, T, y, ldy,
                                           path, None)
     assert call(B=0) == 0                      # empty batch: nothing to do
-    assert call(B=-1) == 1 and call(T=0) == 1 and call(path=4) == 1 and call(x=None) == 1
+    assert call(B=-1) == 1 and call(T=0) == 1 and call(path=5) == 1 and call(x=None) == 1
     assert call(xdt=7) == 4
     assert call(ldx=15) == 2 and call(ldy=15) == 2
     assert call(x=ODD) == 3 and call(codes=ODD) == 3
@@ -119,6 +119,13 @@ def test_wl_matmul_group_validation(lib):
     assert call(ldx=15) == 2 and call(ldy=15) == 2
     assert call(codes=arr(GOOD, ODD, GOOD, GOOD)) == 3        # a misaligned member
     assert call(ys=arr(GOOD, GOOD, None, GOOD)) == 1          # a null member
+    # the group call with an explicit kernel: only paths 0, 1 and 4 exist for a group
+    cp = arr(*([GOOD] * 4))
+    for path in (2, 3, 5, -1):
+        assert lib.fairy2i_wl_matmul_group_path(GOOD, 1, 1, 16, 16, 3, cp, cp, 16, 2, cp, 16,
+                                                path, None) == 1
+    assert lib.fairy2i_wl_matmul_group_path(GOOD, 1, 0, 16, 16, 3, cp, cp, 16, 2, cp, 16, 4,
+                                            None) == 0     # empty batch on path 4
 
 
 def test_codes_adjoint_validation(lib):

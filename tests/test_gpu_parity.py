@@ -447,8 +447,9 @@ def test_bounded_wait_latches_timeout_and_context_survives(F):
     (37, 53, 2, 1, 4, torch.float32),         # fp32 x: members on the general path
 ])
 def test_wl_matmul_group_equals_separate_calls(F, out_f, in_f, T, B, count, dtype):
-    """A group of linears on one input gives, bit for bit, the separate calls' results, and
-    every member matches the oracle."""
+    """A group of linears on one input gives the separate calls' results (bit for bit on the
+    warp-MMA decode kernel, within the accumulation tolerance on the automatic path), and every
+    member matches the oracle."""
     n, m = O.complex_dims(out_f, in_f)
     layers = [_random_quantized(n, m, T, seed=41 + 7 * g + out_f) for g in range(count)]
     x = synth.outlier_activations(B, in_f, seed=43 + in_f).to(dtype)
@@ -457,10 +458,18 @@ def test_wl_matmul_group_equals_separate_calls(F, out_f, in_f, T, B, count, dtyp
     scs = [torch.from_numpy(s).to(DEV) for _, s in layers]
     ys = F.wl_matmul_group(xd, cds, scs, out_f)
     singles = [F.wl_matmul(xd, c, s, out_f) for c, s in zip(cds, scs)]
+    # on the warp-MMA decode kernel (path 1) the group launch and the single calls run the same
+    # arithmetic: bit for bit
+    ys1p = F.wl_matmul_group(xd, cds, scs, out_f, path=1)
+    singles1 = [F.wl_matmul(xd, c, s, out_f, path=1) for c, s in zip(cds, scs)]
     assert F.get_status() == 0
     xo = x.float().numpy()
+    if B <= 2 and dtype == torch.bfloat16:     # where the warp-MMA kernel applies
+        for a1, b1 in zip(ys1p, singles1):
+            assert torch.equal(a1, b1)
     for g, (yg, ys1) in enumerate(zip(ys, singles)):
-        assert torch.equal(yg, ys1)
+        # the automatic path may pick another decode kernel for the group than for a member
+        assert torch.allclose(yg, ys1, rtol=1e-5, atol=1e-5 * float(ys1.abs().max()))
         if out_f * in_f <= 4096 * 4096 and g == 0:
             codes, scales = layers[g]
             assert_wl_close(yg.cpu().numpy(), O.wl_matmul(xo, codes, scales, out_f), xo, scales)
