@@ -57,17 +57,39 @@ def peaks():
 # one decoder layer's decode launches (every layer has the same shapes; grouped: q/k/v, o,
 # gate/up, down; ungrouped: seven), and one T = 2 prefill launch of the 4096 -> 11008 layer on
 # 2048 tokens.
-DECODE_DRAM_BYTES_PER_LAYER = 12.621e6 + 4.232e6 + 22.582e6 + 11.323e6
-DECODE_DRAM_BYTES_PER_LAYER_UNGROUPED = 4 * 4.231e6 + 2 * 11.309e6 + 11.323e6
+# Per call of a decoder layer and decode kernel: "fp8" = the warp-MMA kernel, "stream" = the
+# persistent tcgen05 kernel (grouped calls: q/k/v, gate/up).
+DECODE_DRAM_BYTES = {
+    "fp8": {"q,k,v": 12.621e6, "o": 4.232e6, "gate,up": 22.582e6, "down": 11.323e6,
+            "q": 4.231e6, "k": 4.231e6, "v": 4.231e6, "gate": 11.309e6, "up": 11.309e6},
+    "stream": {"q,k,v": 12.641e6, "gate,up": 22.602e6},
+}
 PREFILL_T2_UP_DRAM_BYTES = 28.087e6 + 38.276e6
 
-def decode_traffic(args):
-    """ncu DRAM bytes of one step's decode launches, where a capture of the kernels this run
-    uses exists (the warp-MMA kernel on every call: --decode-path 1); else None."""
-    if args.decode_path != 1 or args.batch != 1:
+def decode_kernel(c, path, sms):
+    """The decode kernel the library runs for a call at batch <= 2: the automatic path takes the
+    persistent tcgen05 kernel when the call's 16-row tiles outnumber the SMs."""
+    if path == 1:
+        return "fp8"
+    if path == 4:
+        return "stream"
+    n = (c["rows"] + 1) // 2
+    return "stream" if len(c["members"]) * ((n + 15) // 16) > sms else "fp8"
+
+
+def decode_traffic(calls, args, sms):
+    """ncu DRAM bytes of one step's decode launches (batch 1), summed per call from captures of
+    the kernels this run uses; None where no capture exists for a call."""
+    if args.batch != 1:
         return None
-    return int((DECODE_DRAM_BYTES_PER_LAYER_UNGROUPED if args.ungrouped
-                else DECODE_DRAM_BYTES_PER_LAYER) * args.layers)
+    total = 0.0
+    for c in calls:
+        name = ",".join(m["name"] for m in c["members"])
+        v = DECODE_DRAM_BYTES[decode_kernel(c, args.decode_path, sms)].get(name)
+        if v is None:
+            return None
+        total += v
+    return int(total)
 
 
 PREFILL_TOKENS = 2048
@@ -314,6 +336,9 @@ def run_ours(args, world, rank, local):
 
     hbm, _, peak_kind = peaks()
     achieved = step_bytes / (ms_step * 1e-3) / 1e9
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    traffic = decode_traffic(calls, args, sms)
+    kernels = sorted({decode_kernel(c, args.decode_path, sms) for c in calls}) if B <= 2 else []
     line = {
         "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_step, 5),
@@ -333,9 +358,11 @@ def run_ours(args, world, rank, local):
         "gpu_launches": launches_per_step * args.steps,
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm,
                      "unit": "GB/s", "frac": round(achieved / hbm, 4),
-                     "traffic": decode_traffic(args),
+                     "traffic": traffic,
                      "peak_kind": f"{peak_kind} hbm_gbs (burst copy)",
-                     "kernel": "wl_matmul decode (all launches of the step)"},
+                     "kernel": "wl_matmul decode (all launches of the step: "
+                               + " + ".join({"fp8": "warp-MMA", "stream": "persistent tcgen05"}[k]
+                                            for k in kernels) + ")"},
         "clocks": clk,
     }
     if not args.no_prefill:

@@ -87,7 +87,8 @@ constexpr int kOffRing = 0;
 constexpr int kOffB = kOffRing + kRingBytes;                      // 112 KB
 constexpr int kOffRed = kOffB + kMaxU * kChunkB;                  // + 50 KB
 constexpr int kOffGather = kOffRed + 128 * 2 * 2 * 4;             // + 2 KB
-constexpr int kOffBar = kOffGather + 2 * kMaxCluster * kPart * 4; // + 16 KB
+constexpr int kOffOut = kOffGather + 2 * kMaxCluster * kPart * 4; // + 16 KB
+constexpr int kOffBar = kOffOut + kPart * 4;                      // + 1 KB
 constexpr int kNumBars = 2 * kMaxStages + 2 * kSets * kSlots + 2 + 2 + 1 + 2 + 2 + kNumAcc;
 constexpr int kOffMisc = kOffBar + kNumBars * 8;
 constexpr int kSmemBytes = kOffMisc + 512 + 1024;                 // + alignment slack
@@ -120,6 +121,21 @@ struct Misc {
   float scl[kMaxGroup][16];      // scales of the group: [linear][(stage, matrix, re/im)]
   float cpart[4][4];             // per epilogue warp: [token][part] partial C
 };
+
+// Bulk copy of `bytes` (a multiple of 16) from this CTA's shared memory to the shared memory of
+// another CTA of the cluster, completing its bytes on an mbarrier there (cluster addresses).
+__device__ __forceinline__ void bulk_copy_to_cluster(uint32_t dst, uint32_t src, uint32_t bytes,
+                                                     uint32_t mbar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+      ::"r"(dst), "r"(src), "r"(bytes), "r"(mbar)
+      : "memory");
+}
+// Waits until the bulk copies this thread issued have read their sources.
+__device__ __forceinline__ void bulk_commit_wait_read() {
+  asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+  asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+}
 
 __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort,
                                               unsigned int* status) {
@@ -218,6 +234,7 @@ __global__ void __launch_bounds__(kThreads, 1) wl_stream_kernel(const Args a) {
   volatile int* abort_flag = &misc->abort;
   float* red = reinterpret_cast<float*>(smem + kOffRed);
   float* gather = reinterpret_cast<float*>(smem + kOffGather);          // [buf][rank][kPart]
+  float* outp = reinterpret_cast<float*>(smem + kOffOut);               // partial sent to rank 0
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int ks = a.ks;
@@ -240,7 +257,6 @@ __global__ void __launch_bounds__(kThreads, 1) wl_stream_kernel(const Args a) {
       else if (i < 2 * kMaxStages + 2 * kSets * kSlots && i >= 2 * kMaxStages) cnt = kIss;
       else if (bars + i == jfull || bars + i == jfull + 1) cnt = kNumAcc;
       else if (bars + i == jfree || bars + i == jfree + 1) cnt = 4;
-      else if (bars + i == gfull || bars + i == gfull + 1) cnt = ks > 1 ? (ks - 1) * kEpiThreads : 1;
       mbar_init(bars + i, cnt);
     }
     if (lane == 0) misc->abort = 0;
@@ -590,19 +606,27 @@ __global__ void __launch_bounds__(kThreads, 1) wl_stream_kernel(const Args a) {
           // the buffer of job i - 2 in rank 0 has been read
           const bool fr = i < 2 || __all_sync(0xffffffffu, wait_or_abort(&gfree[buf], ((i >> 1) - 1) & 1,
                                                                         abort_flag, a.status));
-          if (fr && !*abort_flag) {
-            const uint32_t g0 = smem_u32(gather) + (uint32_t)((buf * kMaxCluster + rank) * kPart) * 4;
+          // Stage the partial, then one bulk copy into rank 0's gather slot, completing on rank 0's
+          // barrier (also after an abort, so that rank 0 never waits for the full second).
+          const bool ok2 = fr && !*abort_flag;
 #pragma unroll
-            for (int it = 0; it < 2; ++it) {
-              const int idx = et + it * kEpiThreads;
-              if (idx < NV) st_cluster_f32(mapa_shared(g0 + idx * 4, 0), vals[it]);
-            }
+          for (int it = 0; it < 2; ++it) {
+            const int idx = et + it * kEpiThreads;
+            if (idx < NV) outp[idx] = ok2 ? vals[it] : 0.f;
           }
-          // arrive even after an abort, so that rank 0 does not wait for the full second
-          mbar_arrive_remote(mapa_shared(smem_u32(&gfull[buf]), 0));
+          fence_proxy_async_smem();
+          named_bar_sync(1, kEpiThreads);
+          if (et == 0) {
+            const uint32_t g0 =
+                smem_u32(gather) + (uint32_t)((buf * kMaxCluster + rank) * kPart) * 4;
+            bulk_copy_to_cluster(mapa_shared(g0, 0), smem_u32(outp), (uint32_t)(NV * 4),
+                                 mapa_shared(smem_u32(&gfull[buf]), 0));
+            bulk_commit_wait_read();   // outp may be written again by the next job
+          }
         } else {
-          // Waited even after an abort: every rank arrives once per job, and rank 0 stays alive
-          // until those remote arrivals (and the partials before them) have landed.
+          // Waited even after an abort: every rank sends its partial once per job, and rank 0
+          // stays alive until those copies have landed.
+          if (et == 0) mbar_arrive_expect_tx(&gfull[buf], (uint32_t)((ks - 1) * NV * 4));
           const bool got2 = __all_sync(0xffffffffu,
                                        mbar_wait_cluster_timed(&gfull[buf], (i >> 1) & 1, kWaitNs)) &&
                             !*abort_flag;
