@@ -172,10 +172,11 @@ __global__ void __launch_bounds__(kThreads, 1) wl_decode_fp8_kernel(const Args a
       mbar_arrive_expect_tx(bar, (uint32_t)(T2 * nc * kTileBytes));
       const int64_t tiles = (a.n + kRows - 1) / kRows;
 #pragma unroll
+      const uint64_t pol = l2_evict_first_policy();   // the codes are read once per launch
       for (int tm = 0; tm < T2; ++tm)
-        bulk_load(smem + (size_t)(tm * a.nchunks + c_begin) * kTileBytes,
-                  codes + ((tm * tiles + tile) * a.nchunks + c_begin) * kTileWords,
-                  (uint32_t)(nc * kTileBytes), bar);
+        bulk_load_hint(smem + (size_t)(tm * a.nchunks + c_begin) * kTileBytes,
+                       codes + ((tm * tiles + tile) * a.nchunks + c_begin) * kTileWords,
+                       (uint32_t)(nc * kTileBytes), bar, pol);
     }
   }
   __syncwarp();

@@ -317,6 +317,7 @@ __global__ void __launch_bounds__(kThreads, 1) wl_stream_kernel(const Args a) {
   } else if (warp == kCopyWarp) {
     // ---------------- code stream: one stage per job, one bulk copy per tile ----------------
     const int tmi = lane / RT, rt = lane % RT;
+    const uint64_t pol = l2_evict_first_policy();   // the codes are read once per launch
     int issued = 0;
     for (int i = 0; i < njobs; ++i) {
       const int st = i % nstages;
@@ -335,8 +336,9 @@ __global__ void __launch_bounds__(kThreads, 1) wl_stream_kernel(const Args a) {
       __syncwarp();
       if (lane < TM * RT && rt < nrt) {
         const int64_t tile = (int64_t)tmi * a.row_tiles + rb * RT + rt;
-        bulk_load(smem + kOffRing + st * stage_bytes + lane * nu * 512,
-                  a.codes[g] + (tile * a.nch + c0) * 128, (uint32_t)(nu * 512), &full[st]);
+        bulk_load_hint(smem + kOffRing + st * stage_bytes + lane * nu * 512,
+                       a.codes[g] + (tile * a.nch + c0) * 128, (uint32_t)(nu * 512), &full[st],
+                       pol);
       }
       issued = i + 1;
     }
