@@ -162,3 +162,26 @@ def test_stream_rejects_outside_its_domain(F):
                           2 * n, path=2)
     assert e.value.code == 1
     assert F.get_status() == 0
+
+
+def test_automatic_path_routes_by_tile_count(F):
+    """The automatic decode path takes the persistent kernel when a call's 16-row tiles outnumber
+    the SMs (here the grouped q/k/v shape: 3 x 128 tiles) and the warp-MMA kernel otherwise (one
+    4096 -> 4096 linear: 128 tiles): bit for bit the results of the explicit paths, both kernels
+    being deterministic."""
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    out_f, in_f, T = 4096, 4096, 2
+    n, m = O.complex_dims(out_f, in_f)
+    assert 3 * ((n + 15) // 16) > sms >= (n + 15) // 16
+    layers = [_random_quantized(n, m, T, seed=81 + g) for g in range(3)]
+    cds = [_upload(c) for c, _ in layers]
+    scs = [torch.from_numpy(s).to(DEV) for _, s in layers]
+    x = synth.outlier_activations(1, in_f, seed=83).to(DEV)
+    auto_group = F.wl_matmul_group(x, cds, scs, out_f)
+    stream_group = F.wl_matmul_group(x, cds, scs, out_f, path=PATH)
+    auto_single = F.wl_matmul(x, cds[0], scs[0], out_f)
+    warp_single = F.wl_matmul(x, cds[0], scs[0], out_f, path=1)
+    assert F.get_status() == 0
+    for a, b in zip(auto_group, stream_group):
+        assert torch.equal(a, b)
+    assert torch.equal(auto_single, warp_single)
