@@ -122,6 +122,17 @@ __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, vo
   latch_status(status, kStatusTimeout);
   return false;
 }
+// The same for the two MMA-issuing threads: they spin, so that a group's MMAs follow its A
+// stores without a suspended thread's wake-up delay (the issuers are the tensor pipe's feed).
+__device__ __forceinline__ bool spin_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort,
+                                              unsigned int* status) {
+  if (mbar_test_wait(bar, parity)) return true;
+  if (*abort) return false;
+  if (mbar_wait_spin(bar, parity, kWaitNs)) return true;
+  *abort = 1;
+  latch_status(status, kStatusTimeout);
+  return false;
+}
 
 template <int T>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -245,13 +256,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       int g = 0;   // running group counter
       const uint32_t dcol = tmem + kColD + e * 128;
       for (int it = 0; it < my_tiles; ++it) {
-        if (it > 0 && !wait_or_abort(dempty, (it - 1) & 1, abort_flag, a.status)) break;
+        if (it > 0 && !spin_or_abort(dempty, (it - 1) & 1, abort_flag, a.status)) break;
         tc_fence_after();
         bool ok = true;
         for (int gi = 0; gi < gpt; ++gi, ++g) {
           const int slot = g % kG;
           const int xst = (it * nch + (gi >> 1)) % kXS;
-          if (!wait_or_abort(&gfull[slot], (g / kG) & 1, abort_flag, a.status)) {
+          if (!spin_or_abort(&gfull[slot], (g / kG) & 1, abort_flag, a.status)) {
             ok = false;
             break;
           }
