@@ -64,7 +64,7 @@ DECODE_DRAM_BYTES = {
             "q": 4.231e6, "k": 4.231e6, "v": 4.231e6, "gate": 11.309e6, "up": 11.309e6},
     "stream": {"q,k,v": 12.641e6, "gate,up": 22.602e6},
 }
-PREFILL_T2_UP_DRAM_BYTES = 28.087e6 + 38.276e6
+PREFILL_T2_UP_DRAM_BYTES = 28.089e6 + 36.948e6
 
 def decode_kernel(c, path, sms):
     """The decode kernel the library runs for a call at batch <= 2: the automatic path takes the
