@@ -197,7 +197,17 @@ GROUPS = (("q", "k", "v"), ("o",), ("gate", "up"), ("down",))   # linears sharin
 
 def build_stack(F, layers: int, B: int, dev, grouped: bool = True):
     """Converts + quantizes every linear of the stack on the GPU; returns the calls of a step:
-    per call the input x and its member linears (one member each when not grouped)."""
+    per call the input x and its member linears (one member each when not grouped). The inputs
+    of all calls are views of one buffer, the outputs of another, so that a step's activations
+    reach the device and its results the host in one copy each."""
+    groups = GROUPS if grouped else tuple((nm,) for g in GROUPS for nm in g)
+    cols_of = {name: cols for (_, _, name, _, cols) in layer_shapes(1)}
+    rows_of = {name: rows for (_, _, name, rows, _) in layer_shapes(1)}
+    x_all = torch.empty(layers * sum(B * cols_of[g[0]] for g in groups), dtype=torch.bfloat16,
+                        device=dev)
+    y_all = torch.empty(layers * sum(B * rows_of[nm] for g in groups for nm in g),
+                        dtype=torch.float32, device=dev)
+    xo = yo = 0
     calls = []
     for L in range(layers):
         lin = {}
@@ -208,21 +218,24 @@ def build_stack(F, layers: int, B: int, dev, grouped: bool = True):
             del R
             codes, scales = F.quantize(U, W, T_STAGES)
             del U, W
-            y = torch.empty((B, rows), dtype=torch.float32, device=dev)
             lin[name] = dict(L=L, name=name, seed=seed, rows=rows, cols=cols, codes=codes,
-                             scales=scales, y=y)
-        groups = GROUPS if grouped else tuple((nm,) for g in GROUPS for nm in g)
+                             scales=scales)
         for g in groups:
             first = lin[g[0]]
-            x = synth.outlier_activations(B, first["cols"], synth.activation_seed(first["seed"], B),
-                                          device=dev)
+            for nm in g:
+                lin[nm]["y"] = y_all[yo:yo + B * lin[nm]["rows"]].view(B, lin[nm]["rows"])
+                yo += B * lin[nm]["rows"]
+            x = x_all[xo:xo + B * first["cols"]].view(B, first["cols"])
+            xo += B * first["cols"]
+            x.copy_(synth.outlier_activations(B, first["cols"],
+                                              synth.activation_seed(first["seed"], B), device=dev))
             calls.append(dict(x=x, rows=first["rows"], cols=first["cols"],
                               members=[lin[nm] for nm in g]))
     torch.cuda.synchronize()
     status = F.get_status()
     if status != 0:
         raise RuntimeError(f"quantize status {status}")
-    return calls
+    return calls, x_all, y_all
 
 
 def call_bytes(c, B):
@@ -248,7 +261,7 @@ def run_ours(args, world, rank, local):
     F.load()
     dev = torch.device("cuda", local)
     B = args.batch
-    calls = build_stack(F, args.layers, B, dev, grouped=not args.ungrouped)
+    calls, x_all, y_all = build_stack(F, args.layers, B, dev, grouped=not args.ungrouped)
     step_bytes = sum(call_bytes(c, B) for c in calls)
     nlinears = sum(len(c["members"]) for c in calls)
     # a grouped call is one launch where the decode kernel takes it (B <= 2), else one per member
@@ -300,19 +313,17 @@ def run_ours(args, world, rank, local):
         raise RuntimeError(f"device status {st} after the timed region")
 
     # end to end through the public call with host buffers: per step the inputs of all
-    # linears go host->device from pinned memory and every output comes back to the host.
-    xs_host = [c["x"].cpu().pin_memory() for c in calls]
-    ys_dev = [m["y"] for c in calls for m in c["members"]]
-    ys_host = [torch.empty(y.shape, dtype=torch.float32).pin_memory() for y in ys_dev]
-    h2d = sum(x.numel() * x.element_size() for x in xs_host)
-    d2h = sum(y.numel() * 4 for y in ys_host)
+    # linears go host->device from pinned memory and every output comes back to the host (one
+    # copy each way: the calls' inputs and outputs are views of x_all and y_all).
+    x_host = x_all.cpu().pin_memory()
+    y_host = torch.empty(y_all.shape, dtype=torch.float32).pin_memory()
+    h2d = x_host.numel() * x_host.element_size()
+    d2h = y_host.numel() * 4
 
     def e2e_step():
-        for c, xh in zip(calls, xs_host):
-            c["x"].copy_(xh, non_blocking=True)
+        x_all.copy_(x_host, non_blocking=True)
         run()
-        for y, yh in zip(ys_dev, ys_host):
-            yh.copy_(y, non_blocking=True)
+        y_host.copy_(y_all, non_blocking=True)
 
     with torch.cuda.stream(stream):
         for _ in range(args.warmup):
@@ -366,7 +377,7 @@ def run_ours(args, world, rank, local):
         "clocks": clk,
     }
     if not args.no_prefill:
-        del calls, ys_dev
+        del calls, x_all, y_all
         torch.cuda.empty_cache()
         line["prefill"] = run_prefill(F, dev, args.prefill_steps, max(args.warmup, 3))
     if rank == 0 and not args.no_cpu_baseline:

@@ -150,6 +150,20 @@ __device__ __forceinline__ bool mbar_wait_spin(uint64_t* bar, uint32_t parity, u
   }
 }
 
+// Polling form for waits on the critical path of a pipeline: non-blocking tests with a short
+// sleep between them, so the thread resumes within ~100 cycles of the phase completing (a
+// suspended try_wait resumes hundreds of cycles later) without taking many issue slots.
+__device__ __forceinline__ bool mbar_wait_poll(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
+  if (mbar_test_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  const long long limit = (long long)(limit_ns * 5 / 2);
+  for (;;) {
+    __nanosleep(32);
+    if (mbar_test_wait(bar, parity)) return true;
+    if (clock64() - t0 > limit) return false;
+  }
+}
+
 // ---- plain mbarrier arrive, named barriers ----
 __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
   asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar))

@@ -140,7 +140,7 @@ __device__ __forceinline__ void bulk_commit_wait_read() {
 __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort,
                                               unsigned int* status) {
   if (*abort) return false;
-  if (mbar_wait_timed(bar, parity, kWaitNs)) return true;
+  if (mbar_wait_poll(bar, parity, kWaitNs)) return true;
   *abort = 1;
   latch_status(status, kStatusTimeout);
   return false;
