@@ -90,6 +90,28 @@ __device__ __forceinline__ void mma_e4m3_ts(uint32_t d_tmem, uint32_t a_tmem, ui
       "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
+// Instruction descriptor of kind::mxf4 (block-scaled e2m1 x e2m1, f32 accumulate, K = 64):
+// A and B format E2M1 (1) in bits 7-9 and 10-11, K-major A and B, N >> 3 at bit 17, scale
+// factors UE8M0 (bit 23), M >> 4 at bit 24, scale-factor byte selectors 0.
+__host__ __device__ constexpr uint32_t idesc_mxf4_f32(int M, int N) {
+  return (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | (1u << 23) |
+         ((uint32_t)(M >> 4) << 24);
+}
+
+// D[tmem] (+)= A[tmem] * B[smem]^T with packed e2m1 operands (two per byte, the lower K index in
+// the low nibble; A row m in TMEM lane m, K index k at nibble k % 8 of column k / 8) and one
+// ue8m0 scale factor per 32 K values of every row of A and B, read from TMEM at sfa and sfb.
+__device__ __forceinline__ void mma_mxf4_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
+                                            uint32_t idesc, uint32_t sfa, uint32_t sfb,
+                                            uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %6, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::mxf4.block_scale.scale_vec::2X [%0], [%1], %2, %3, [%4], "
+      "[%5], p;\n}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(sfa), "r"(sfb), "r"(accumulate)
+      : "memory");
+}
+
 // Arrive once on `bar` when every tcgen05 operation this thread issued before has completed.
 __device__ __forceinline__ void mma_commit(uint64_t* bar) {
   asm volatile(

@@ -1,6 +1,6 @@
 // Persistent decode (B <= 2 tokens) kernel of the quantized widely-linear matmul on the
 // 5th-generation tensor cores: the packed codes stream through shared memory, are decoded into
-// tensor memory and multiplied there (tcgen05.mma, kind::f8f6f4, A in TMEM).
+// tensor memory and multiplied there (tcgen05.mma with A in TMEM).
 //
 // Arithmetic (Eq. ifairy-dequant, Algorithm 1 with the W conj(x) term). Every code carries the
 // signs sigma = sign(Re b + Im b), tau = sign(Re b - Im b) of its codeword b; with
@@ -9,13 +9,23 @@
 // h conj(P) + conj(h) conj(Q) for W (the conj(x) term of Eq. widely-linear).
 //
 // Tensor-core form. TMEM lane L = tm R + r holds row r of stage-matrix tm = 2 t + matrix
-// (R = 64, 32, 16, 16 rows for T = 1..4). One MMA (M = 128, N = 16, K = 32, e4m3 x e4m3 -> f32)
-// covers one code word (16 codes) of the 128 lanes. A word becomes 32 A bytes, (sigma_2j,
-// sigma_2j+1, tau_2j, tau_2j+1) for j = 0..7, each an e4m3 value affine in its bit by one LOP3
-// per four bytes (a = alpha + 2 bit, sigma = (1 + alpha) - a), so P = C - D, D the MMA result
-// and C = sum_k (1 + alpha_k) x_k the same for every row. B holds x split exactly into two e4m3
-// limbs (hi = e4m3(x S), lo = e4m3(64 (x S - hi)), S a power of two per CTA and token) in the
-// 16 columns (token, limb, sigma/tau slot, re/im).
+// (R = 64, 32, 16, 16 rows for T = 1..4); an MMA has M = 128 and accumulates in f32. The time
+// of one MMA follows the bytes of A it reads from TMEM, not N, so A is kept small and x is
+// spread over the N columns.
+// * One token: kind::mxf4 (e2m1 x e2m1, unit ue8m0 scale factors), K = 64. A code word (16
+//   codes) becomes four A registers of eight nibbles, +1 = 0x2 or -1 = 0xA, four sigma and four
+//   tau each (one shift and one LOP3 per register), so one MMA covers two words. x is X = rn(|x| S) < 2^24 (S a power of two per CTA) in twelve base-4
+//   digits d_l, held as the e2m1 values +-d_l / 2 with the sign of x, in the 48 columns
+//   (slot, re/im, limb): the sigma slot has them at the sigma positions of K and zeros at the
+//   tau positions, the tau slot the reverse. The sums of digits are exact in f32, and
+//   P = (2 / S) sum_l 4^l D_l.
+// * Two tokens: kind::f8f6f4 (e4m3), K = 32, one MMA per word. A word becomes 32 A bytes
+//   (sigma_2j, sigma_2j+1, tau_2j, tau_2j+1) for j = 0..7, each an e4m3 value affine in its bit
+//   by one LOP3 per four bytes (a = alpha + 2 bit, sigma = (1 + alpha) - a), so P = C - D, D the
+//   MMA result and C = sum_k (1 + alpha_k) x_k the same for every row. B holds x split exactly
+//   into two e4m3 limbs (hi = e4m3(x S), lo = e4m3(64 (x S - hi)), S a power of two per CTA and
+//   token) in the 16 columns (token, limb, sigma/tau slot, re/im). The e2m1 form of two tokens
+//   would need 96 accumulator columns per set.
 //
 // Work. A job is one row block (R rows of every stage-matrix) of one linear of the group; the
 // jobs are dealt round-robin to thread-block clusters of ks CTAs, and rank r of a cluster takes
@@ -32,12 +42,12 @@
 // the copies of the codes into the shared-memory ring and their decoding into tensor memory
 // start before griddepcontrol.wait; the B tiles, and with them every MMA, come after it.
 //
-// Roles (17 warps): warps 0-7 are two decoder sets of four (warp w reaches TMEM lanes
-// 32 (w % 4) ..), set s decoding units q = s, s + 2, ... into its three A slots; warp 8 streams
-// the codes; lane 0 of warp 9 + 2 s + e issues the MMAs of words 4e .. 4e + 3 of every unit of
-// set s into its own accumulator of the job's buffer (two buffers, so a job's read-out overlaps
-// the next job's MMAs); warps 13-16 load x, build the B tiles, C and S, then read out, combine
-// and reduce every job's accumulators and write y.
+// Roles: warps 0-7 are two decoder sets of four (warp w reaches TMEM lanes 32 (w % 4) ..), set s
+// decoding units q = s, s + 2, ... into its three A slots; warp 8 streams the codes; lane 0 of
+// warp 9 + s (e2m1) or of warps 9 + 2 s + e (e4m3: words 4e .. 4e + 3) issues the MMAs of every
+// unit of set s into its own accumulator of the job's buffer (two buffers, so a job's read-out
+// overlaps the next job's MMAs); the last four warps load x, build the B tiles (and C) and S,
+// then read out, combine and reduce every job's accumulators and write y.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
@@ -54,48 +64,62 @@ namespace fairy2i {
 namespace sd {
 
 constexpr int kSets = 2;                      // decoder sets of four warps
-constexpr int kSlots = 3;                     // A slots per set (one unit, 64 TMEM columns)
-constexpr int kIss = 2;                       // MMA-issuing threads per set (words 0-3, 4-7)
 constexpr int kDecWarps = 4 * kSets;          // warps 0-7
 constexpr int kCopyWarp = kDecWarps;          // 8
-constexpr int kIssWarp0 = kCopyWarp + 1;      // 9-12: warp kIssWarp0 + kIss s + e
-constexpr int kEpiWarp0 = kIssWarp0 + kSets * kIss;   // 13-16 (warp % 4 = 1, 2, 3, 0)
-constexpr int kWarps = kEpiWarp0 + 4;         // 17
-constexpr int kThreads = kWarps * 32;         // 544
+constexpr int kIssWarp0 = kCopyWarp + 1;      // warp kIssWarp0 + kIss s + e
 constexpr int kEpiThreads = 128;
 constexpr int kRingBytes = 112 * 1024;        // code ring: one job (nu units) per stage
 constexpr int kMaxStages = 14;
 constexpr int kUnitBytes = 4096;              // codes of one unit (8 tiles x 512 B)
-constexpr int kWordB = 528;                   // B tile of one word: 16 rows x 32 bytes, + 16 B
-                                              // so that the tiles of consecutive words start in
-                                              // different shared-memory banks
-constexpr int kChunkB = 8 * kWordB;           // B tiles of one chunk
 constexpr int kMaxU = 12;                     // chunks per CTA
 constexpr int kMaxCluster = 8;
 constexpr int kMaxGroup = 4;
 constexpr int kPart = 256;                    // floats of one partial (R rows x NB x 2)
-constexpr int kAccCols = 16;
-constexpr int kNumAcc = kSets * kIss;         // accumulators per job buffer
-constexpr int kColSlots = 2 * kNumAcc * kAccCols;   // accumulators: [buffer][set][issuer] x 16
 constexpr int kTmemCols = 512;
 constexpr uint64_t kWaitNs = 1000000000ull;   // 1 s: a pipeline wait is microseconds
-constexpr uint32_t kIdesc = idesc_e4m3_f32(128, 16);
-static_assert(kColSlots + kSets * kSlots * 64 <= kTmemCols, "TMEM columns");
+constexpr int kLimbs4 = 12;                   // base-4 digits of x in the e2m1 form
 
-// Shared memory layout (bytes from the 1024-aligned base).
-constexpr int kOffRing = 0;
-constexpr int kOffB = kOffRing + kRingBytes;                      // 112 KB
-constexpr int kOffRed = kOffB + kMaxU * kChunkB;                  // + 50 KB
-constexpr int kOffGather = kOffRed + 128 * 2 * 2 * 4;             // + 2 KB
-constexpr int kOffOut = kOffGather + 2 * kMaxCluster * kPart * 4; // + 16 KB
-constexpr int kOffBar = kOffOut + kPart * 4;                      // + 1 KB
-constexpr int kNumBars = 2 * kMaxStages + 2 * kSets * kSlots + 2 + 2 + 1 + 2 + 2 + kNumAcc;
-constexpr int kOffMisc = kOffBar + kNumBars * 8;
-constexpr int kSmemBytes = kOffMisc + 512 + 1024;                 // + alignment slack
-// One CTA per SM: it owns all TMEM columns (a second CTA on the SM would wait in its allocation),
-// and no two CTAs of a launch share an SM's tensor core.
-static_assert(kSmemBytes > 116 * 1024, "one CTA per SM");
-static_assert(kSmemBytes <= 227 * 1024, "shared memory per CTA");
+// Operand form and layout. One token (NB = 1): e2m1 (kind::mxf4), two codes' signs per A byte,
+// one MMA (K = 64) per two code words, x as kLimbs4 base-4 digits in 48 B columns (slot, part,
+// limb); one issuing thread per set. Two tokens: e4m3 (kind::f8f6f4), one MMA (K = 32) per
+// word, x as two e4m3 limbs in 16 B columns (token, limb, slot, part); two issuing threads per
+// set (words 0-3, 4-7). The e2m1 form of two tokens would need 96 accumulator columns per set.
+template <int NB>
+struct Layout {
+  static constexpr bool kF4 = NB == 1;
+  static constexpr int kSlots = 3;                          // A slots per set (one unit each)
+  static constexpr int kIss = kF4 ? 1 : 2;                  // MMA-issuing threads per set
+  static constexpr int kNumAcc = kSets * kIss;              // accumulators per job buffer
+  static constexpr int kN = kF4 ? 2 * 2 * kLimbs4 : 16;     // MMA N (B columns)
+  static constexpr int kAccStride = kF4 ? 64 : 16;          // TMEM columns per accumulator
+  static constexpr int kColSlots = 2 * kNumAcc * kAccStride;   // accumulators [buffer][set][issuer]
+  static constexpr int kSlotCols = kF4 ? 32 : 64;           // TMEM columns of one unit's A
+  static constexpr int kColSF = kColSlots + kSets * kSlots * kSlotCols;   // scale factors (e2m1)
+  static constexpr int kMmas = kF4 ? 4 : 8;                 // MMAs per unit
+  // B tile of one MMA: kN rows x 32 bytes, + 16 B so that consecutive tiles start in different
+  // shared-memory banks.
+  static constexpr int kMmaB = kN * 32 + 16;
+  static constexpr int kChunkB = kMmas * kMmaB;             // B tiles of one chunk
+  static constexpr uint32_t kIdesc = kF4 ? idesc_mxf4_f32(128, kN) : idesc_e4m3_f32(128, kN);
+  static constexpr int kEpiWarp0 = kIssWarp0 + kSets * kIss;   // four warps, every warp % 4
+  static constexpr int kWarps = kEpiWarp0 + 4;
+  static constexpr int kThreads = kWarps * 32;
+  // Shared memory (bytes from the 1024-aligned base).
+  static constexpr int kOffRing = 0;
+  static constexpr int kOffB = kOffRing + kRingBytes;
+  static constexpr int kOffRed = kOffB + kMaxU * kChunkB;
+  static constexpr int kOffGather = kOffRed + 128 * 2 * 2 * 4;
+  static constexpr int kOffOut = kOffGather + 2 * kMaxCluster * kPart * 4;
+  static constexpr int kOffBar = kOffOut + kPart * 4;
+  static constexpr int kNumBars = 2 * kMaxStages + 2 * kSets * kSlots + 2 + 2 + 1 + 2 + 2 + kNumAcc;
+  static constexpr int kOffMisc = kOffBar + kNumBars * 8;
+  static constexpr int kSmemBytes = kOffMisc + 512 + 1024;   // + alignment slack
+  static_assert(kColSF + (kF4 ? 64 : 0) <= kTmemCols, "TMEM columns");
+  // One CTA per SM: it owns all TMEM columns (a second CTA on the SM would wait in its
+  // allocation), and no two CTAs of a launch share an SM's tensor core.
+  static_assert(kSmemBytes > 116 * 1024, "one CTA per SM");
+  static_assert(kSmemBytes <= 227 * 1024, "shared memory per CTA");
+};
 
 struct Args {
   const uint32_t* codes[kMaxGroup];
@@ -161,6 +185,18 @@ __device__ __forceinline__ void decode_word(uint32_t w0, uint32_t* r) {
   r[7] = lop3_and_xor(w0, 0x80808080u, 0xB8B8B8B8u);
 }
 
+// e2m1 form: the four A registers of a word. The word holds the sign bits of sigma in bits 0-15
+// and of tau in bits 16-31, code i at bit 8 (i % 2) + i / 2 of its half. Register s keeps the
+// bits 4 n + 3 - s of the word as the sign bits (4 n + 3) of nibbles n = 0..7 on the magnitude
+// 1 (0x2): nibbles 0-3 are sigma and nibbles 4-7 tau of the codes at bits 4 n + 3 - s of the
+// halves (0x2 = +1, 0xA = -1). One shift and one LOP3 per register.
+__device__ __forceinline__ void decode_word4(uint32_t w, uint32_t* r) {
+  r[0] = lop3_and_or(w, 0x88888888u, 0x22222222u);
+  r[1] = lop3_and_or(w << 1, 0x88888888u, 0x22222222u);
+  r[2] = lop3_and_or(w << 2, 0x88888888u, 0x22222222u);
+  r[3] = lop3_and_or(w << 3, 0x88888888u, 0x22222222u);
+}
+
 __device__ __forceinline__ float bf_lo(uint32_t v) { return __uint_as_float(v << 16); }
 __device__ __forceinline__ float bf_hi(uint32_t v) { return __uint_as_float(v & 0xffff0000u); }
 
@@ -209,7 +245,16 @@ __device__ __forceinline__ void job_of(const Args& a, int cluster, int i, int& g
 }
 
 template <int NB, int T>
-__global__ void __launch_bounds__(kThreads, 1) wl_stream_kernel(const Args a) {
+__global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(const Args a) {
+  using Lay = Layout<NB>;
+  constexpr bool kF4 = Lay::kF4;
+  constexpr int kSlots = Lay::kSlots, kIss = Lay::kIss, kNumAcc = Lay::kNumAcc;
+  constexpr int kEpiWarp0 = Lay::kEpiWarp0;
+  constexpr int kColSlots = Lay::kColSlots, kSlotCols = Lay::kSlotCols;
+  constexpr int kAccStride = Lay::kAccStride, kMmaB = Lay::kMmaB, kChunkB = Lay::kChunkB;
+  constexpr int kOffRing = Lay::kOffRing, kOffB = Lay::kOffB, kOffRed = Lay::kOffRed;
+  constexpr int kOffGather = Lay::kOffGather, kOffOut = Lay::kOffOut, kOffBar = Lay::kOffBar;
+  constexpr int kOffMisc = Lay::kOffMisc, kNumBars = Lay::kNumBars;
   constexpr int TM = 2 * T;
   constexpr int R = (T == 1) ? 64 : (T == 2 ? 32 : 16);  // rows per row block
   constexpr int RT = R / 16;                              // 16-row code tiles per row block
@@ -266,8 +311,23 @@ __global__ void __launch_bounds__(kThreads, 1) wl_stream_kernel(const Args a) {
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  if (ks > 1) cluster_arrive();   // barriers of every rank initialised (waited before DSMEM use)
   const uint32_t tmem = misc->tmem;
+  if constexpr (kF4) {
+    // Unit scale factors (ue8m0 127 = 1.0) for every row of A and B of every MMA.
+    if (warp < 4) {
+      uint32_t ones[32];
+#pragma unroll
+      for (int i = 0; i < 32; ++i) ones[i] = 0x7F7F7F7Fu;
+      const uint32_t la = tmem + ((uint32_t)(warp * 32) << 16) + Lay::kColSF;
+      tmem_st32(la, ones);
+      tmem_st32(la + 32, ones);
+      tmem_wait_st();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+  }
+  if (ks > 1) cluster_arrive();   // barriers of every rank initialised (waited before DSMEM use)
   pdl_launch_dependents();
 
   if (warp < kDecWarps) {
@@ -279,12 +339,26 @@ __global__ void __launch_bounds__(kThreads, 1) wl_stream_kernel(const Args a) {
     const uint32_t lane_off = (uint32_t)((tm * RT + r / 16) * nu * 512 + (r % 16) * 32);
     const uint32_t ring = smem_u32(smem + kOffRing);
     const uint32_t t_lane = tmem + ((uint32_t)(quarter * 32) << 16) + kColSlots;
+    // unit q = set + kSets l: chunk u of job i, in ring stage st (its (i / nstages)-th use,
+    // phase fph) and A slot sl of the set (its (l / kSlots)-th use, phase ph); no divisions
+    int i = 0, u = set, st = 0, sl = 0;
+    uint32_t fph = 0, ph = 0;
+    auto next_job = [&]() {
+      ++i;
+      if (++st == nstages) {
+        st = 0;
+        fph ^= 1u;
+      }
+    };
+    while (u >= nu) {
+      u -= nu;
+      next_job();
+    }
     int l = 0;
     for (int q = set; q < total; q += kSets, ++l) {
-      const int i = q / nu, u = q - i * nu;
-      const int st = i % nstages, sl = l % kSlots, si = set * kSlots + sl;
-      if (!__all_sync(0xffffffffu, wait_or_abort(&full[st], (i / nstages) & 1, abort_flag,
-                                                  a.status)))
+      const int si = set * kSlots + sl;
+      if (!__all_sync(0xffffffffu, mbar_test_wait(&full[st], fph) ||
+                                       wait_or_abort(&full[st], fph, abort_flag, a.status)))
         break;
       const uint32_t src = ring + st * stage_bytes + lane_off + u * 512;
       const uint4 q0 = lds128(src), q1 = lds128(src + 16);
@@ -294,25 +368,46 @@ __global__ void __launch_bounds__(kThreads, 1) wl_stream_kernel(const Args a) {
       // that no bounded wait below counts its run time.
       if (l == kSlots) pdl_wait_primary();
       if (l >= kSlots &&   // the slot's previous unit has been multiplied
-          !__all_sync(0xffffffffu, wait_or_abort(&sfree[si], ((l / kSlots) - 1) & 1, abort_flag,
-                                                  a.status)))
+          !__all_sync(0xffffffffu, mbar_test_wait(&sfree[si], ph ^ 1u) ||
+                                       wait_or_abort(&sfree[si], ph ^ 1u, abort_flag, a.status)))
         break;
-      const uint32_t a_col = t_lane + si * 64;
+      const uint32_t a_col = t_lane + si * kSlotCols;
       uint32_t rr[32];
-      decode_word(q0.x, rr);
-      decode_word(q0.y, rr + 8);
-      decode_word(q0.z, rr + 16);
-      decode_word(q0.w, rr + 24);
-      tmem_st32(a_col, rr);
-      decode_word(q1.x, rr);
-      decode_word(q1.y, rr + 8);
-      decode_word(q1.z, rr + 16);
-      decode_word(q1.w, rr + 24);
-      tmem_st32(a_col + 32, rr);
+      if constexpr (kF4) {   // word w -> columns 4 w .. 4 w + 3
+        decode_word4(q0.x, rr);
+        decode_word4(q0.y, rr + 4);
+        decode_word4(q0.z, rr + 8);
+        decode_word4(q0.w, rr + 12);
+        decode_word4(q1.x, rr + 16);
+        decode_word4(q1.y, rr + 20);
+        decode_word4(q1.z, rr + 24);
+        decode_word4(q1.w, rr + 28);
+        tmem_st32(a_col, rr);
+      } else {               // word w -> columns 8 w .. 8 w + 7
+        decode_word(q0.x, rr);
+        decode_word(q0.y, rr + 8);
+        decode_word(q0.z, rr + 16);
+        decode_word(q0.w, rr + 24);
+        tmem_st32(a_col, rr);
+        decode_word(q1.x, rr);
+        decode_word(q1.y, rr + 8);
+        decode_word(q1.z, rr + 16);
+        decode_word(q1.w, rr + 24);
+        tmem_st32(a_col + 32, rr);
+      }
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&sfull[si]);
+      if (++sl == kSlots) {
+        sl = 0;
+        ph ^= 1u;
+      }
+      u += kSets;
+      while (u >= nu) {
+        u -= nu;
+        next_job();
+      }
     }
   } else if (warp == kCopyWarp) {
     // ---------------- code stream: one stage per job, one bulk copy per tile ----------------
@@ -357,15 +452,24 @@ __global__ void __launch_bounds__(kThreads, 1) wl_stream_kernel(const Args a) {
       bool ok = wait_or_abort(bready, 0, abort_flag, a.status);
       tc_fence_after();
       bool issued = false;
-      int l = 0, cur = -1;
+      int cur = -1;
       bool first = true;
       // Before touching job i's accumulator buffer, the read-out of job i - 2 must be done; a
       // job without a unit of this set still gets this issuer's arrival.
       auto enter_job = [&](int i) {
         if (i >= 2 && ok) ok = wait_or_abort(&jfree[i & 1], ((i >> 1) - 1) & 1, abort_flag, a.status);
       };
-      for (int q = set; ok && q < total; q += kSets, ++l) {
-        const int i = q / nu, u = q - i * nu;
+      // Unit q = set + kSets l of the CTA is chunk u of job i, in slot sl of the set for the
+      // (l / kSlots)-th time (phase ph); advanced without divisions, since this thread's loop
+      // overhead adds to every unit.
+      int i = 0, u = set, sl = 0;
+      uint32_t ph = 0;
+      while (u >= nu) {
+        u -= nu;
+        ++i;
+      }
+      const uint64_t desc0 = smem_desc(b_base, 128, 256);   // + (byte offset >> 4) per tile
+      for (int q = set; ok && q < total; q += kSets) {
         if (i != cur) {
           if (cur >= 0) mma_commit(&jfull[cur & 1]);
           for (int i2 = cur + 1; ok && i2 < i; ++i2) {   // jobs without a unit of this set
@@ -378,22 +482,38 @@ __global__ void __launch_bounds__(kThreads, 1) wl_stream_kernel(const Args a) {
           cur = i;
           first = true;
         }
-        const int si = set * kSlots + l % kSlots;
-        ok = wait_or_abort(&sfull[si], (l / kSlots) & 1, abort_flag, a.status);
+        const int si = set * kSlots + sl;
+        ok = mbar_test_wait(&sfull[si], ph) || wait_or_abort(&sfull[si], ph, abort_flag, a.status);
         if (!ok) break;
         tc_fence_after();
-        const uint32_t a_slot = tmem + kColSlots + si * 64;
-        const uint32_t d_tmem = tmem + ((cur & 1) * kNumAcc + ii) * kAccCols;
-        const uint32_t bt = b_base + u * kChunkB;
+        const uint32_t a_slot = tmem + kColSlots + si * kSlotCols;
+        const uint32_t d_tmem = tmem + ((cur & 1) * kNumAcc + ii) * kAccStride;
+        const uint64_t bd = desc0 + (uint64_t)((u * kChunkB) >> 4);
+        if constexpr (kF4) {   // MMA j: words 2 j, 2 j + 1 (A columns 8 j ..)
 #pragma unroll
-        for (int w4 = 0; w4 < 4; ++w4) {
-          const int w = e * 4 + w4;
-          mma_e4m3_ts(d_tmem, a_slot + w * 8, smem_desc(bt + w * kWordB, 128, 256), kIdesc,
-                      (first && w4 == 0) ? 0u : 1u);
+          for (int j = 0; j < 4; ++j)
+            mma_mxf4_ts(d_tmem, a_slot + j * 8, bd + (uint64_t)((j * kMmaB) >> 4), Lay::kIdesc,
+                        tmem + Lay::kColSF, tmem + Lay::kColSF + 16, (first && j == 0) ? 0u : 1u);
+        } else {               // MMA w: word w (A columns 8 w ..)
+#pragma unroll
+          for (int w4 = 0; w4 < 4; ++w4) {
+            const int w = e * 4 + w4;
+            mma_e4m3_ts(d_tmem, a_slot + w * 8, bd + (uint64_t)((w * kMmaB) >> 4), Lay::kIdesc,
+                        (first && w4 == 0) ? 0u : 1u);
+          }
         }
         first = false;
         issued = true;
         mma_commit(&sfree[si]);
+        if (++sl == kSlots) {
+          sl = 0;
+          ph ^= 1u;
+        }
+        u += kSets;
+        while (u >= nu) {
+          u -= nu;
+          ++i;
+        }
       }
       if (ok) {
         if (cur >= 0) mma_commit(&jfull[cur & 1]);
@@ -418,8 +538,9 @@ __global__ void __launch_bounds__(kThreads, 1) wl_stream_kernel(const Args a) {
     const int64_t kbeg = (int64_t)c0 * 128;
     // Before the wait: zero the B tiles (rows of unused tokens stay zero) and warm L2 with the
     // x slice.
-    for (int o = et; o < nu * kChunkB / 16; o += kEpiThreads)
-      *reinterpret_cast<uint4*>(smem + kOffB + o * 16) = make_uint4(0, 0, 0, 0);
+    if constexpr (!kF4)   // (the e2m1 tiles are written whole)
+      for (int o = et; o < nu * kChunkB / 16; o += kEpiThreads)
+        *reinterpret_cast<uint4*>(smem + kOffB + o * 16) = make_uint4(0, 0, 0, 0);
     // the scales, like the codes, are not written by the previous kernel
     if (et < a.G * TM * 2) misc->scl[et / (TM * 2)][et % (TM * 2)] = __ldg(a.scales[et / (TM * 2)] + et % (TM * 2));
     if (a.x_bulk && et < 2 * NB && et / 2 < a.B) {
@@ -431,105 +552,189 @@ __global__ void __launch_bounds__(kThreads, 1) wl_stream_kernel(const Args a) {
                          (uint32_t)((k1 - kbeg) * 2));
     }
     pdl_wait_primary();               // x may be written by the previous kernel
-    // This thread's groups: for token b and part p, the 8-value groups v = et + 128 jv of the
-    // slice (v < 16 nu), values x_p[8 v .. 8 v + 7].
-    constexpr int kJv = 2;                      // 16 kMaxU / 128 groups per (b, p) and thread
-    static_assert(16 * kMaxU <= kJv * kEpiThreads, "x groups per thread");
-    uint4 xv[NB][2][kJv];
+    // e4m3: x S in two limbs, P = C - D; e2m1: X = |x| S in base-4 digits
+    float S[2] = {1.f, 1.f}, invS[2] = {1.f, 1.f}, C[4] = {0.f, 0.f, 0.f, 0.f};
+    if constexpr (kF4) {
+      // Items it = (8 u + w) 2 + p of the slice: the 16 values x_p[kbeg + 128 u + 16 w + i],
+      // i = 0..15, of code word w of chunk u (two items per thread at most).
+      static_assert(16 * kMaxU <= 2 * kEpiThreads, "x items per thread");
+      uint4 xv[2][2];
 #pragma unroll
-    for (int b = 0; b < NB; ++b)
-#pragma unroll
-      for (int p = 0; p < 2; ++p)
-#pragma unroll
-        for (int jv = 0; jv < kJv; ++jv) {
-          const int v = et + jv * kEpiThreads;
-          xv[b][p][jv] = (v < nu * 16 && b < a.B) ? load_x8(a, b, p, kbeg + v * 8)
-                                                  : make_uint4(0, 0, 0, 0);
+      for (int j = 0; j < 2; ++j) {
+        const int it = et + j * kEpiThreads;
+        xv[j][0] = xv[j][1] = make_uint4(0, 0, 0, 0);
+        if (it < nu * 16) {
+          const int64_t k = kbeg + 128 * (it >> 4) + 16 * ((it >> 1) & 7);
+          xv[j][0] = load_x8(a, 0, it & 1, k);
+          xv[j][1] = load_x8(a, 0, it & 1, k + 8);
         }
-    // max |x| per token (non-negative float bits order like unsigned integers)
+      }
+      unsigned int mx = 0u;   // max |x| (non-negative float bits order like unsigned integers)
 #pragma unroll
-    for (int b = 0; b < NB; ++b) {
-      unsigned int mx = 0u;
+      for (int j = 0; j < 2; ++j)
 #pragma unroll
-      for (int p = 0; p < 2; ++p)
-#pragma unroll
-        for (int jv = 0; jv < kJv; ++jv) {
-          const uint32_t ev[4] = {xv[b][p][jv].x, xv[b][p][jv].y, xv[b][p][jv].z, xv[b][p][jv].w};
+        for (int h = 0; h < 2; ++h) {
+          const uint32_t ev[4] = {xv[j][h].x, xv[j][h].y, xv[j][h].z, xv[j][h].w};
 #pragma unroll
           for (int i = 0; i < 4; ++i) mx = max(mx, max((ev[i] << 17) >> 1, ev[i] & 0x7fff0000u));
         }
       mx = __reduce_max_sync(0xffffffffu, mx);
-      if (lane == 0) misc->xmax[ew][b] = mx;
-    }
-    named_bar_sync(1, kEpiThreads);
-    float S[2] = {1.f, 1.f}, invS[2] = {1.f, 1.f};
+      if (lane == 0) misc->xmax[ew][0] = mx;
+      named_bar_sync(1, kEpiThreads);
+      const unsigned int xm = max(max(misc->xmax[0][0], misc->xmax[1][0]),
+                                  max(misc->xmax[2][0], misc->xmax[3][0]));
+      // S = 2^(24 - E) for 2^(E-1) <= max|x| < 2^E: every X = rn(|x| S) < 2^24 is kLimbs4
+      // base-4 digits, and P = (2 / S) sum_l 4^l D_l with D_l the MMA column of digit l (e2m1
+      // holds digit d as d / 2).
+      const int se = min(254, max(1, 277 - (int)(xm >> 23)));
+      S[0] = __uint_as_float((uint32_t)se << 23);
+      invS[0] = 2.f / S[0];
 #pragma unroll
-    for (int b = 0; b < NB; ++b) {
-      const unsigned int xm = max(max(misc->xmax[0][b], misc->xmax[1][b]),
-                                  max(misc->xmax[2][b], misc->xmax[3][b]));
-      pow2_scale(__uint_as_float(xm), S[b], invS[b]);
-    }
-    // B tiles and C. Group v = 16 u + 2 w + hh of token b, part p: the values x_p[k], k = 128 u +
-    // 16 w + 8 hh .. + 7, become the 16-byte halves hh of the four rows (limb, slot, p) of token b
-    // in the tile of word w of chunk u: register j' (codes 2j, 2j + 1, j = 4 hh + j') holds the
-    // limb bytes of x[2j], x[2j + 1] in its sigma half (bytes 0-1) or tau half (bytes 2-3).
-    float cacc[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
+      for (int j = 0; j < 2; ++j) {
+        const int it = et + j * kEpiThreads;
+        if (it < nu * 16) {
+          const int u = it >> 4, w = (it >> 1) & 7, p = it & 1;
+          // register i of the item: codes 2 i (low half) and 2 i + 1 (high half)
+          const uint32_t ev[8] = {xv[j][0].x, xv[j][0].y, xv[j][0].z, xv[j][0].w,
+                                  xv[j][1].x, xv[j][1].y, xv[j][1].z, xv[j][1].w};
+          uint32_t xc[16], sg[16];   // X and sign of code c of the word
 #pragma unroll
-    for (int b = 0; b < NB; ++b)
+          for (int i = 0; i < 8; ++i) {
+            xc[2 * i] = __float2uint_rn(fabsf(bf_lo(ev[i])) * S[0]);
+            xc[2 * i + 1] = __float2uint_rn(fabsf(bf_hi(ev[i])) * S[0]);
+            sg[2 * i] = (ev[i] >> 15) & 1u;
+            sg[2 * i + 1] = ev[i] >> 31;
+          }
+          // Row (slot, p, l) of the MMA tile of words 2 (w / 2), + 1, half w % 2: A register s
+          // of the word pairs nibble n (n < 4) with sigma, nibble n + 4 with tau of the code at
+          // bit q = 4 n + 3 - s of a half (code 2 q, or 2 (q - 8) + 1 for q >= 8). The sigma
+          // slot holds digit l of x of that code in nibble n of word s, the tau slot in nibble
+          // n + 4.
+          unsigned char* tile = smem + kOffB + u * kChunkB + (w >> 1) * kMmaB + (w & 1) * 128;
 #pragma unroll
-      for (int p = 0; p < 2; ++p)
+          for (int l = 0; l < kLimbs4; ++l) {
+            uint32_t ws[4];
 #pragma unroll
-        for (int jv = 0; jv < kJv; ++jv) {
-          const int v = et + jv * kEpiThreads;
-          if (v < nu * 16) {
-            const int u = v >> 4, w = (v >> 1) & 7, hh = v & 1;
-            const uint32_t ev[4] = {xv[b][p][jv].x, xv[b][p][jv].y, xv[b][p][jv].z,
-                                    xv[b][p][jv].w};
-            uint32_t hp[4], lp[4];   // limb byte pairs (x[2j], x[2j+1]) of register j'
-            float cs = 0.f;
+            for (int sh = 0; sh < 4; ++sh) {
+              ws[sh] = 0u;
 #pragma unroll
-            for (int jj = 0; jj < 4; ++jj) {
-              const float f0 = bf_lo(ev[jj]), f1 = bf_hi(ev[jj]);
-              const float v0 = f0 * S[b], v1 = f1 * S[b];
-              hp[jj] = e4m3x2(v0, v1) & 0xffffu;
-              const float2 hf = e4m3x2_to_float2(hp[jj]);
-              lp[jj] = e4m3x2(64.f * (v0 - hf.x), 64.f * (v1 - hf.y)) & 0xffffu;
-              // 1 + alpha of codes 2j, 2j+1: 5, 3, 5, 3 (first half of a word), 1, 0, 1, 0
-              const float wgt = hh ? ((jj & 1) ? 0.f : 1.f) : ((jj & 1) ? 3.f : 5.f);
-              cs = fmaf(wgt, f0 + f1, cs);
+              for (int nn = 0; nn < 4; ++nn) {
+                const int q = 4 * nn + 3 - sh;
+                const int c = q < 8 ? 2 * q : 2 * (q - 8) + 1;
+                ws[sh] |= (((xc[c] >> (2 * l)) & 3u) | (sg[c] << 3)) << (4 * nn);
+              }
             }
-            cacc[b][p] += cs;
-            unsigned char* tile = smem + kOffB + u * kChunkB + w * kWordB;
+            const int ns = p * kLimbs4 + l, nt = (2 + p) * kLimbs4 + l;
+            *reinterpret_cast<uint4*>(tile + (ns >> 3) * 256 + (ns & 7) * 16) =
+                make_uint4(ws[0], ws[1], ws[2], ws[3]);
+            *reinterpret_cast<uint4*>(tile + (nt >> 3) * 256 + (nt & 7) * 16) =
+                make_uint4(ws[0] << 16, ws[1] << 16, ws[2] << 16, ws[3] << 16);
+          }
+        }
+      }
+      fence_proxy_async_smem();   // generic-proxy writes of B visible to the tensor cores
+      named_bar_sync(1, kEpiThreads);
+      if (et == 0) mbar_arrive(bready);
+    } else {
+      // This thread's groups: for token b and part p, the 8-value groups v = et + 128 jv of the
+      // slice (v < 16 nu), values x_p[8 v .. 8 v + 7].
+      constexpr int kJv = 2;                      // 16 kMaxU / 128 groups per (b, p) and thread
+      static_assert(16 * kMaxU <= kJv * kEpiThreads, "x groups per thread");
+      uint4 xv[NB][2][kJv];
 #pragma unroll
-            for (int limb = 0; limb < 2; ++limb) {
-              const uint32_t* src = limb ? lp : hp;
+      for (int b = 0; b < NB; ++b)
 #pragma unroll
-              for (int slot = 0; slot < 2; ++slot) {
-                const int nrow = ((b * 2 + limb) * 2 + slot) * 2 + p;
-                const int sh = slot ? 16 : 0;
-                *reinterpret_cast<uint4*>(tile + (nrow >> 3) * 256 + hh * 128 + (nrow & 7) * 16) =
-                    make_uint4(src[0] << sh, src[1] << sh, src[2] << sh, src[3] << sh);
+        for (int p = 0; p < 2; ++p)
+#pragma unroll
+          for (int jv = 0; jv < kJv; ++jv) {
+            const int v = et + jv * kEpiThreads;
+            xv[b][p][jv] = (v < nu * 16 && b < a.B) ? load_x8(a, b, p, kbeg + v * 8)
+                                                    : make_uint4(0, 0, 0, 0);
+          }
+      // max |x| per token (non-negative float bits order like unsigned integers)
+#pragma unroll
+      for (int b = 0; b < NB; ++b) {
+        unsigned int mx = 0u;
+#pragma unroll
+        for (int p = 0; p < 2; ++p)
+#pragma unroll
+          for (int jv = 0; jv < kJv; ++jv) {
+            const uint32_t ev[4] = {xv[b][p][jv].x, xv[b][p][jv].y, xv[b][p][jv].z, xv[b][p][jv].w};
+#pragma unroll
+            for (int i = 0; i < 4; ++i) mx = max(mx, max((ev[i] << 17) >> 1, ev[i] & 0x7fff0000u));
+          }
+        mx = __reduce_max_sync(0xffffffffu, mx);
+        if (lane == 0) misc->xmax[ew][b] = mx;
+      }
+      named_bar_sync(1, kEpiThreads);
+#pragma unroll
+      for (int b = 0; b < NB; ++b) {
+        const unsigned int xm = max(max(misc->xmax[0][b], misc->xmax[1][b]),
+                                    max(misc->xmax[2][b], misc->xmax[3][b]));
+        pow2_scale(__uint_as_float(xm), S[b], invS[b]);
+      }
+      // B tiles and C. Group v = 16 u + 2 w + hh of token b, part p: the values x_p[k], k = 128 u +
+      // 16 w + 8 hh .. + 7, become the 16-byte halves hh of the four rows (limb, slot, p) of token b
+      // in the tile of word w of chunk u: register j' (codes 2j, 2j + 1, j = 4 hh + j') holds the
+      // limb bytes of x[2j], x[2j + 1] in its sigma half (bytes 0-1) or tau half (bytes 2-3).
+      float cacc[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
+#pragma unroll
+      for (int b = 0; b < NB; ++b)
+#pragma unroll
+        for (int p = 0; p < 2; ++p)
+#pragma unroll
+          for (int jv = 0; jv < kJv; ++jv) {
+            const int v = et + jv * kEpiThreads;
+            if (v < nu * 16) {
+              const int u = v >> 4, w = (v >> 1) & 7, hh = v & 1;
+              const uint32_t ev[4] = {xv[b][p][jv].x, xv[b][p][jv].y, xv[b][p][jv].z,
+                                      xv[b][p][jv].w};
+              uint32_t hp[4], lp[4];   // limb byte pairs (x[2j], x[2j+1]) of register j'
+              float cs = 0.f;
+#pragma unroll
+              for (int jj = 0; jj < 4; ++jj) {
+                const float f0 = bf_lo(ev[jj]), f1 = bf_hi(ev[jj]);
+                const float v0 = f0 * S[b], v1 = f1 * S[b];
+                hp[jj] = e4m3x2(v0, v1) & 0xffffu;
+                const float2 hf = e4m3x2_to_float2(hp[jj]);
+                lp[jj] = e4m3x2(64.f * (v0 - hf.x), 64.f * (v1 - hf.y)) & 0xffffu;
+                // 1 + alpha of codes 2j, 2j+1: 5, 3, 5, 3 (first half of a word), 1, 0, 1, 0
+                const float wgt = hh ? ((jj & 1) ? 0.f : 1.f) : ((jj & 1) ? 3.f : 5.f);
+                cs = fmaf(wgt, f0 + f1, cs);
+              }
+              cacc[b][p] += cs;
+              unsigned char* tile = smem + kOffB + u * kChunkB + w * kMmaB;
+#pragma unroll
+              for (int limb = 0; limb < 2; ++limb) {
+                const uint32_t* src = limb ? lp : hp;
+#pragma unroll
+                for (int slot = 0; slot < 2; ++slot) {
+                  const int nrow = ((b * 2 + limb) * 2 + slot) * 2 + p;
+                  const int sh = slot ? 16 : 0;
+                  *reinterpret_cast<uint4*>(tile + (nrow >> 3) * 256 + hh * 128 + (nrow & 7) * 16) =
+                      make_uint4(src[0] << sh, src[1] << sh, src[2] << sh, src[3] << sh);
+                }
               }
             }
           }
+      fence_proxy_async_smem();   // generic-proxy writes of B visible to the tensor cores
+      named_bar_sync(1, kEpiThreads);
+      if (et == 0) mbar_arrive(bready);
+#pragma unroll
+      for (int b = 0; b < 2; ++b)
+#pragma unroll
+        for (int p = 0; p < 2; ++p) {
+          float v = cacc[b][p];
+#pragma unroll
+          for (int h = 16; h >= 1; h >>= 1) v += __shfl_xor_sync(0xffffffffu, v, h);
+          if (lane == 0) misc->cpart[ew][b * 2 + p] = v;
         }
-    fence_proxy_async_smem();   // generic-proxy writes of B visible to the tensor cores
-    named_bar_sync(1, kEpiThreads);
-    if (et == 0) mbar_arrive(bready);
+      named_bar_sync(1, kEpiThreads);
 #pragma unroll
-    for (int b = 0; b < 2; ++b)
-#pragma unroll
-      for (int p = 0; p < 2; ++p) {
-        float v = cacc[b][p];
-#pragma unroll
-        for (int h = 16; h >= 1; h >>= 1) v += __shfl_xor_sync(0xffffffffu, v, h);
-        if (lane == 0) misc->cpart[ew][b * 2 + p] = v;
-      }
-    named_bar_sync(1, kEpiThreads);
-    float C[4];
-#pragma unroll
-    for (int j = 0; j < 4; ++j)
-      C[j] = (misc->cpart[0][j] + misc->cpart[1][j]) + (misc->cpart[2][j] + misc->cpart[3][j]);
+      for (int j = 0; j < 4; ++j)
+        C[j] = (misc->cpart[0][j] + misc->cpart[1][j]) + (misc->cpart[2][j] + misc->cpart[3][j]);
+
+    }
 
     // ---- per job: read out, combine with the scales, sum the stage-matrices, reduce ----
     if (ks > 1) cluster_wait();   // every rank's barriers are initialised
@@ -538,26 +743,50 @@ __global__ void __launch_bounds__(kThreads, 1) wl_stream_kernel(const Args a) {
       const int buf = i & 1;
       int g, rb;
       job_of(a, cluster, i, g, rb);
-      float d[16];
+      float d[16];   // e4m3: columns (token, limb, slot, part)
 #pragma unroll
       for (int k = 0; k < 16; ++k) d[k] = 0.f;
+      float d4[4] = {0.f, 0.f, 0.f, 0.f};   // e2m1: sum_l 4^l D_l of (slot, part)
       const bool got = __all_sync(0xffffffffu,
                                   wait_or_abort(&jfull[buf], (i >> 1) & 1, abort_flag, a.status));
       tc_fence_after();
+      // sets with at least one unit in job i
+      auto has = [&](int s) { return nu >= kSets || ((s - i * nu) % kSets + kSets) % kSets < nu; };
+      const uint32_t acc0 = tmem + ((uint32_t)(quarter * 32) << 16) + buf * kNumAcc * kAccStride;
       if (got) {
+        if constexpr (kF4) {
 #pragma unroll
-        for (int s = 0; s < kSets; ++s) {
-          // sets with at least one unit in job i
-          const bool has = nu >= kSets || ((s - i * nu) % kSets + kSets) % kSets < nu;
-          if (has) {
-            float v0[16], v1[16];
-            const uint32_t acc = tmem + ((uint32_t)(quarter * 32) << 16) +
-                                 (buf * kNumAcc + s * kIss) * kAccCols;
-            tmem_ld16(acc, v0);
-            tmem_ld16(acc + kAccCols, v1);
+          for (int c16 = 0; c16 < Lay::kN / 16; ++c16) {
+            float v[kSets][16];
+#pragma unroll
+            for (int s = 0; s < kSets; ++s) {
+              if (has(s)) {
+                tmem_ld16(acc0 + s * kAccStride + c16 * 16, v[s]);
+              } else {
+#pragma unroll
+                for (int k = 0; k < 16; ++k) v[s][k] = 0.f;
+              }
+            }
             tmem_wait_ld();
 #pragma unroll
-            for (int k = 0; k < 16; ++k) d[k] += v0[k] + v1[k];
+            for (int k = 0; k < 16; ++k) {
+              const int col = c16 * 16 + k;   // (slot 2 + part) kLimbs4 + limb
+              d4[col / kLimbs4] = fmaf(v[0][k] + v[1][k], (float)(1u << (2 * (col % kLimbs4))),
+                                       d4[col / kLimbs4]);
+            }
+          }
+        } else {
+#pragma unroll
+          for (int s = 0; s < kSets; ++s) {
+            if (has(s)) {
+              float v0[16], v1[16];
+              const uint32_t acc = acc0 + s * kIss * kAccStride;
+              tmem_ld16(acc, v0);
+              tmem_ld16(acc + kAccStride, v1);
+              tmem_wait_ld();
+#pragma unroll
+              for (int k = 0; k < 16; ++k) d[k] += v0[k] + v1[k];
+            }
           }
         }
       }
@@ -569,6 +798,17 @@ __global__ void __launch_bounds__(kThreads, 1) wl_stream_kernel(const Args a) {
         const bool mat = tmL & 1;
         const float hr = 0.5f * misc->scl[g][(t * 2 + mat) * 2 + 0];
         const float hi = 0.5f * misc->scl[g][(t * 2 + mat) * 2 + 1];
+        if constexpr (kF4) {
+          const float is = invS[0];
+          const float pre = d4[0] * is, qre = d4[2] * is;
+          float pim = d4[1] * is, qim = d4[3] * is;
+          if (mat) {   // W multiplies conj(x): conjugate P and Q
+            pim = -pim;
+            qim = -qim;
+          }
+          red[L * 2 + 0] = hr * pre - hi * pim + hr * qre + hi * qim;
+          red[L * 2 + 1] = hr * pim + hi * pre + hr * qim - hi * qre;
+        } else {
 #pragma unroll
         for (int b = 0; b < NB; ++b) {
           const float cre = C[b * 2 + 0], cim = C[b * 2 + 1];
@@ -585,6 +825,7 @@ __global__ void __launch_bounds__(kThreads, 1) wl_stream_kernel(const Args a) {
           }
           red[(L * NB + b) * 2 + 0] = hr * pre - hi * pim + hr * qre + hi * qim;
           red[(L * NB + b) * 2 + 1] = hr * pim + hi * pre + hr * qim - hi * qre;
+        }
         }
       }
       named_bar_sync(1, kEpiThreads);
@@ -687,15 +928,15 @@ fairy2i_status launch(const Args& a, int64_t grid, cudaStream_t stream) {
   auto kern = wl_stream_kernel<NB, T>;
   static bool configured = false;
   if (!configured) {
-    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) !=
-        cudaSuccess)
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             Layout<NB>::kSmemBytes) != cudaSuccess)
       return FAIRY2I_ERR_CUDA;
     configured = true;
   }
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)grid);
-  cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.blockDim = dim3(Layout<NB>::kThreads);
+  cfg.dynamicSmemBytes = Layout<NB>::kSmemBytes;
   cfg.stream = stream;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -714,13 +955,13 @@ fairy2i_status launch(const Args& a, int64_t grid, cudaStream_t stream) {
 template <int NB, int T>
 int max_clusters(int ks) {
   auto kern = wl_stream_kernel<NB, T>;
-  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) !=
-      cudaSuccess)
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           Layout<NB>::kSmemBytes) != cudaSuccess)
     return 0;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)(ks * 256));
-  cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.blockDim = dim3(Layout<NB>::kThreads);
+  cfg.dynamicSmemBytes = Layout<NB>::kSmemBytes;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = (unsigned)ks;
