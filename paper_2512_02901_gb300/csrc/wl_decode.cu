@@ -149,9 +149,21 @@ __global__ void __launch_bounds__(kThreads, 1) wl_decode_fp8_kernel(const Args a
   extern __shared__ __align__(1024) unsigned char smem[];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int g = lane >> 2, t4 = lane & 3;
-  const int lin = (int)blockIdx.x / a.tiles, tile = (int)blockIdx.x - lin * a.tiles;
+  int lin = 0, tile = (int)blockIdx.x;   // linear of the group and row tile (count <= 4)
+  while (tile >= a.tiles) {
+    tile -= a.tiles;
+    ++lin;
+  }
   const uint32_t* const codes = a.codes[lin];
   const float* const scales = a.scales[lin];
+  // The scales, like the codes, are not written by the previous kernel: read them now, so that
+  // their latency is not paid after the MMAs.
+  float scl[T2][2];
+#pragma unroll
+  for (int tm = 0; tm < T2; ++tm) {
+    scl[tm][0] = __ldg(scales + tm * 2 + 0);
+    scl[tm][1] = __ldg(scales + tm * 2 + 1);
+  }
   const int64_t j0 = (int64_t)tile * kRows;
   const uint32_t* codes_s = reinterpret_cast<const uint32_t*>(smem);
   uint64_t* bar = reinterpret_cast<uint64_t*>(smem + a.bar_off) + warp;
@@ -312,8 +324,8 @@ __global__ void __launch_bounds__(kThreads, 1) wl_decode_fp8_kernel(const Args a
   float sre_u = 0.f, sre_w = 0.f;
 #pragma unroll
   for (int t = 0; t < T; ++t) {
-    sre_u += __ldg(scales + (t * 2 + 0) * 2);
-    sre_w += __ldg(scales + (t * 2 + 1) * 2);
+    sre_u += scl[t * 2 + 0][0];
+    sre_w += scl[t * 2 + 1][0];
   }
 #pragma unroll
   for (int b = 0; b < NB; ++b) {
@@ -323,8 +335,8 @@ __global__ void __launch_bounds__(kThreads, 1) wl_decode_fp8_kernel(const Args a
 #pragma unroll
     for (int tm = 0; tm < T2; ++tm) {
       const int t = tm >> 1, mat = tm & 1;
-      const float hr = 0.5f * __ldg(scales + (t * 2 + mat) * 2 + 0);
-      const float hs = 0.5f * __ldg(scales + (t * 2 + mat) * 2 + 1);
+      const float hr = 0.5f * scl[t * 2 + mat][0];
+      const float hs = 0.5f * scl[t * 2 + mat][1];
       const float hi = is_q ? -hs : hs;          // conj(h) multiplies Q
       const float di0 = mat ? -acc[b][tm][1] : acc[b][tm][1];   // W multiplies conj(x)
       const float di1 = mat ? -acc[b][tm][3] : acc[b][tm][3];

@@ -111,7 +111,7 @@ struct Layout {
   static constexpr int kOffGather = kOffRed + 128 * 2 * 2 * 4;
   static constexpr int kOffOut = kOffGather + 2 * kMaxCluster * kPart * 4;
   static constexpr int kOffBar = kOffOut + kPart * 4;
-  static constexpr int kNumBars = 2 * kMaxStages + 2 * kSets * kSlots + 2 + 2 + 1 + 2 + 2 + kNumAcc;
+  static constexpr int kNumBars = 2 * kMaxStages + 2 * kSets * kSlots + 2 + 2 + 1 + 2 + 2 + kNumAcc + 1;
   static constexpr int kOffMisc = kOffBar + kNumBars * 8;
   static constexpr int kSmemBytes = kOffMisc + 512 + 1024;   // + alignment slack
   static_assert(kColSF + (kF4 ? 64 : 0) <= kTmemCols, "TMEM columns");
@@ -275,6 +275,7 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
   uint64_t* gfull = bready + 1;                 // [buffer] rank 0: partials arrived
   uint64_t* gfree = gfull + 2;                  // [buffer] ranks > 0: rank 0 read the buffer
   uint64_t* fin = gfree + 2;                    // [issuer] abort path
+  uint64_t* sfready = fin + kNumAcc;            // e2m1: scale factors written (4 warps)
   Misc* misc = reinterpret_cast<Misc*>(smem + kOffMisc);
   volatile int* abort_flag = &misc->abort;
   float* red = reinterpret_cast<float*>(smem + kOffRed);
@@ -302,6 +303,7 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
       else if (i < 2 * kMaxStages + 2 * kSets * kSlots && i >= 2 * kMaxStages) cnt = kIss;
       else if (bars + i == jfull || bars + i == jfull + 1) cnt = kNumAcc;
       else if (bars + i == jfree || bars + i == jfree + 1) cnt = 4;
+      else if (bars + i == sfready) cnt = 4;
       mbar_init(bars + i, cnt);
     }
     if (lane == 0) misc->abort = 0;
@@ -312,20 +314,19 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = misc->tmem;
-  if constexpr (kF4) {
-    // Unit scale factors (ue8m0 127 = 1.0) for every row of A and B of every MMA.
-    if (warp < 4) {
-      uint32_t ones[32];
+  if (kF4 && warp < 4) {
+    // Unit scale factors (ue8m0 127 = 1.0) for every row of A and B of every MMA; the issuing
+    // threads wait for them on sfready (off the other roles' path).
+    uint32_t ones[32];
 #pragma unroll
-      for (int i = 0; i < 32; ++i) ones[i] = 0x7F7F7F7Fu;
-      const uint32_t la = tmem + ((uint32_t)(warp * 32) << 16) + Lay::kColSF;
-      tmem_st32(la, ones);
-      tmem_st32(la + 32, ones);
-      tmem_wait_st();
-    }
+    for (int i = 0; i < 32; ++i) ones[i] = 0x7F7F7F7Fu;
+    const uint32_t la = tmem + ((uint32_t)(warp * 32) << 16) + Lay::kColSF;
+    tmem_st32(la, ones);
+    tmem_st32(la + 32, ones);
+    tmem_wait_st();
     tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(sfready);
   }
   if (ks > 1) cluster_arrive();   // barriers of every rank initialised (waited before DSMEM use)
   pdl_launch_dependents();
@@ -450,6 +451,7 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
       const uint32_t b_base = smem_u32(smem + kOffB);
       pdl_wait_primary();   // the B tiles are built from x after the previous kernel
       bool ok = wait_or_abort(bready, 0, abort_flag, a.status);
+      if (kF4 && ok) ok = wait_or_abort(sfready, 0, abort_flag, a.status);
       tc_fence_after();
       bool issued = false;
       int cur = -1;
@@ -542,7 +544,8 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
       for (int o = et; o < nu * kChunkB / 16; o += kEpiThreads)
         *reinterpret_cast<uint4*>(smem + kOffB + o * 16) = make_uint4(0, 0, 0, 0);
     // the scales, like the codes, are not written by the previous kernel
-    if (et < a.G * TM * 2) misc->scl[et / (TM * 2)][et % (TM * 2)] = __ldg(a.scales[et / (TM * 2)] + et % (TM * 2));
+    // (stored into shared memory after the B tiles: the load's latency stays off the path to x)
+    const float scl_v = et < a.G * TM * 2 ? __ldg(a.scales[et / (TM * 2)] + et % (TM * 2)) : 0.f;
     if (a.x_bulk && et < 2 * NB && et / 2 < a.B) {
       const int b = et >> 1, p = et & 1;
       const int64_t lim = p ? a.in_features - a.m : a.m;
@@ -632,6 +635,7 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
           }
         }
       }
+      if (et < a.G * TM * 2) misc->scl[et / (TM * 2)][et % (TM * 2)] = scl_v;
       fence_proxy_async_smem();   // generic-proxy writes of B visible to the tensor cores
       named_bar_sync(1, kEpiThreads);
       if (et == 0) mbar_arrive(bready);
@@ -717,6 +721,7 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
               }
             }
           }
+      if (et < a.G * TM * 2) misc->scl[et / (TM * 2)][et % (TM * 2)] = scl_v;
       fence_proxy_async_smem();   // generic-proxy writes of B visible to the tensor cores
       named_bar_sync(1, kEpiThreads);
       if (et == 0) mbar_arrive(bready);
