@@ -165,8 +165,9 @@ fairy2i_status fairy2i_wl_matmul(const void* x, fairy2i_dtype xdt, int64_t B,
  *   4 = the persistent tcgen05 decode kernel (one CTA per SM looping over row blocks, the codes
  *       streamed through shared memory and decoded into tensor memory, K split over thread-block
  *       clusters of up to 8 CTAs whose partial rows are summed in rank order; one token: e2m1
- *       operands, x held to 2^-24 of the largest |x| in a CTA's part of the K range; two
- *       tokens: e4m3 operands, x as two e4m3 limbs); it takes B <= 2 bf16 tokens, T <= 4 and
+ *       operands, each x entry held to 2^-26 of the largest |x| in a CTA's part of the K range,
+ *       which keeps every output within the per-element bound for any x; two tokens: e4m3
+ *       operands, x as two e4m3 limbs); it takes B <= 2 bf16 tokens, T <= 4 and
  *       in_features <= 24576 and returns FAIRY2I_ERR_INVALID_ARG for anything else.
  * The decode kernels (paths 1, 2, 4) read the codes and scales before waiting for the previous
  * kernel in the stream (programmatic dependent launch): the codes must not be written by the

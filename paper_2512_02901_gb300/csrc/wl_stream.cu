@@ -14,11 +14,11 @@
 // spread over the N columns.
 // * One token: kind::mxf4 (e2m1 x e2m1, unit ue8m0 scale factors), K = 64. A code word (16
 //   codes) becomes four A registers of eight nibbles, +1 = 0x2 or -1 = 0xA, four sigma and four
-//   tau each (one shift and one LOP3 per register), so one MMA covers two words. x is X = rn(|x| S) < 2^24 (S a power of two per CTA) in twelve base-4
-//   digits d_l, held as the e2m1 values +-d_l / 2 with the sign of x, in the 48 columns
-//   (slot, re/im, limb): the sigma slot has them at the sigma positions of K and zeros at the
-//   tau positions, the tau slot the reverse. The sums of digits are exact in f32, and
-//   P = (2 / S) sum_l 4^l D_l.
+//   tau each (one shift and one LOP3 per register), so one MMA covers two words. x is
+//   X = rn(|x| S) < 2^26 (S a power of two per CTA) in thirteen base-4 digits d_l, held as the
+//   e2m1 values +-d_l / 2 with the sign of x, in the first 52 of 64 columns (slot, re/im, limb):
+//   the sigma slot has them at the sigma positions of K and zeros at the tau positions, the tau
+//   slot the reverse. The sums of digits are exact in f32, and P = (2 / S) sum_l 4^l D_l.
 // * Two tokens: kind::f8f6f4 (e4m3), K = 32, one MMA per word. A word becomes 32 A bytes
 //   (sigma_2j, sigma_2j+1, tau_2j, tau_2j+1) for j = 0..7, each an e4m3 value affine in its bit
 //   by one LOP3 per four bytes (a = alpha + 2 bit, sigma = (1 + alpha) - a), so P = C - D, D the
@@ -74,14 +74,17 @@ constexpr int kUnitBytes = 4096;              // codes of one unit (8 tiles x 51
 constexpr int kMaxU = 12;                     // chunks per CTA
 constexpr int kMaxCluster = 8;
 constexpr int kMaxGroup = 4;
-constexpr int kPart = 256;                    // floats of one partial (R rows x NB x 2)
 constexpr int kTmemCols = 512;
 constexpr uint64_t kWaitNs = 1000000000ull;   // 1 s: a pipeline wait is microseconds
-constexpr int kLimbs4 = 12;                   // base-4 digits of x in the e2m1 form
+// Base-4 digits of x in the e2m1 form: 2^-26 of the largest |x| of a CTA's K slice (at most
+// 2 kMaxU 128 = 3072 real values) bounds the error of every x entry, so the x error in l1 norm
+// stays below 3072 2^-26 = 4.6e-5 of |x|_1, within the 1e-4 |x|_1 sum_t s_t bound per output
+// for any input.
+constexpr int kLimbs4 = 13;
 
 // Operand form and layout. One token (NB = 1): e2m1 (kind::mxf4), two codes' signs per A byte,
-// one MMA (K = 64) per two code words, x as kLimbs4 base-4 digits in 48 B columns (slot, part,
-// limb); one issuing thread per set. Two tokens: e4m3 (kind::f8f6f4), one MMA (K = 32) per
+// one MMA (K = 64) per two code words, x as kLimbs4 base-4 digits in the first 52 of 64 B
+// columns (slot, part, limb); one issuing thread per set. Two tokens: e4m3 (kind::f8f6f4), one MMA (K = 32) per
 // word, x as two e4m3 limbs in 16 B columns (token, limb, slot, part); two issuing threads per
 // set (words 0-3, 4-7). The e2m1 form of two tokens would need 96 accumulator columns per set.
 template <int NB>
@@ -90,7 +93,9 @@ struct Layout {
   static constexpr int kSlots = 3;                          // A slots per set (one unit each)
   static constexpr int kIss = kF4 ? 1 : 2;                  // MMA-issuing threads per set
   static constexpr int kNumAcc = kSets * kIss;              // accumulators per job buffer
-  static constexpr int kN = kF4 ? 2 * 2 * kLimbs4 : 16;     // MMA N (B columns)
+  static constexpr int kNUsed = kF4 ? 2 * 2 * kLimbs4 : 16; // B columns holding x
+  static constexpr int kN = (kNUsed + 15) / 16 * 16;        // MMA N (the rest zero)
+  static constexpr int kPart = 128 * NB;                    // floats of one partial (R NB 2)
   static constexpr int kAccStride = kF4 ? 64 : 16;          // TMEM columns per accumulator
   static constexpr int kColSlots = 2 * kNumAcc * kAccStride;   // accumulators [buffer][set][issuer]
   static constexpr int kSlotCols = kF4 ? 32 : 64;           // TMEM columns of one unit's A
@@ -260,6 +265,7 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
   constexpr int RT = R / 16;                              // 16-row code tiles per row block
   constexpr int NV = R * NB * 2;                          // outputs of a row block
   static_assert(TM * RT * 512 <= kUnitBytes, "unit size");
+  constexpr int kPart = Lay::kPart;
   static_assert(NV <= kPart && NV <= 2 * kEpiThreads, "partial size");
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>(
@@ -540,9 +546,17 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
     const int64_t kbeg = (int64_t)c0 * 128;
     // Before the wait: zero the B tiles (rows of unused tokens stay zero) and warm L2 with the
     // x slice.
-    if constexpr (!kF4)   // (the e2m1 tiles are written whole)
+    if constexpr (!kF4) {
       for (int o = et; o < nu * kChunkB / 16; o += kEpiThreads)
         *reinterpret_cast<uint4*>(smem + kOffB + o * 16) = make_uint4(0, 0, 0, 0);
+    } else {   // the rows past the digits, 16 bytes (row, half) at a time
+      constexpr int kSpare = (Lay::kN - Lay::kNUsed) * 2;
+      for (int o = et; o < nu * Lay::kMmas * kSpare; o += kEpiThreads) {
+        const int tile = o / kSpare, rest = o % kSpare, n = Lay::kNUsed + (rest >> 1);
+        *reinterpret_cast<uint4*>(smem + kOffB + tile * kMmaB + (n >> 3) * 256 + (rest & 1) * 128 +
+                                  (n & 7) * 16) = make_uint4(0, 0, 0, 0);
+      }
+    }
     // the scales, like the codes, are not written by the previous kernel
     // (stored into shared memory after the B tiles: the load's latency stays off the path to x)
     const float scl_v = et < a.G * TM * 2 ? __ldg(a.scales[et / (TM * 2)] + et % (TM * 2)) : 0.f;
@@ -586,10 +600,10 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
       named_bar_sync(1, kEpiThreads);
       const unsigned int xm = max(max(misc->xmax[0][0], misc->xmax[1][0]),
                                   max(misc->xmax[2][0], misc->xmax[3][0]));
-      // S = 2^(24 - E) for 2^(E-1) <= max|x| < 2^E: every X = rn(|x| S) < 2^24 is kLimbs4
+      // S = 2^(26 - E) for 2^(E-1) <= max|x| < 2^E: every X = rn(|x| S) < 2^26 is kLimbs4
       // base-4 digits, and P = (2 / S) sum_l 4^l D_l with D_l the MMA column of digit l (e2m1
       // holds digit d as d / 2).
-      const int se = min(254, max(1, 277 - (int)(xm >> 23)));
+      const int se = min(254, max(1, 127 + 2 * kLimbs4 + 126 - (int)(xm >> 23)));
       S[0] = __uint_as_float((uint32_t)se << 23);
       invS[0] = 2.f / S[0];
 #pragma unroll
@@ -776,8 +790,9 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
 #pragma unroll
             for (int k = 0; k < 16; ++k) {
               const int col = c16 * 16 + k;   // (slot 2 + part) kLimbs4 + limb
-              d4[col / kLimbs4] = fmaf(v[0][k] + v[1][k], (float)(1u << (2 * (col % kLimbs4))),
-                                       d4[col / kLimbs4]);
+              if (col < Lay::kNUsed)
+                d4[col / kLimbs4] = fmaf(v[0][k] + v[1][k], (float)(1u << (2 * (col % kLimbs4))),
+                                         d4[col / kLimbs4]);
             }
           }
         } else {

@@ -185,3 +185,26 @@ def test_automatic_path_routes_by_tile_count(F):
     for a, b in zip(auto_group, stream_group):
         assert torch.equal(a, b)
     assert torch.equal(auto_single, warp_single)
+
+
+@pytest.mark.parametrize("tiny", [0.99609375 * 2.0**-24, 0.99609375 * 2.0**-26])
+def test_stream_one_token_element_bound_for_extreme_x(F, tiny):
+    """The one-token form holds each x entry to half a unit in 2^-26 of the largest |x| of the
+    CTA's K slice, so the l1 error of x stays below 3072 2^-26 |x|_1 (a slice holds at most 3072
+    real values) and the error of every output below the per-element bound 1e-4 |x~|_1 sum_t s_t,
+    whatever x is. Worst case here: 152 row blocks of 1536-input rows (one CTA takes a whole row),
+    x = (1, tiny, tiny, ...) with the tiny entries just under half a unit (2^-24 would fall off
+    with twelve digits), every code +1 so that the errors add up in every row. The relative
+    Frobenius criterion is not checked: no fixed precision meets it for every input."""
+    T, out_f, in_f = 2, 9728, 3072
+    n, m = O.complex_dims(out_f, in_f)
+    codes = np.zeros((T, 2, n, m), dtype=np.uint8)
+    scales = np.full((T, 2, 2), 0.02, dtype=np.float32)
+    x = torch.full((1, in_f), tiny, dtype=torch.float32).to(torch.bfloat16)
+    x[0, 0] = 1.0
+    y = F.wl_matmul(x.to(DEV), _upload(codes), torch.from_numpy(scales).to(DEV), out_f, path=PATH)
+    assert F.get_status() == 0
+    xo = x.float().numpy().astype(np.float64)
+    err = np.asarray(y.cpu().numpy(), np.float64) - O.wl_matmul(xo, codes, scales, out_f)
+    bound = 1e-4 * O.tolerance_bound(xo, scales)[:, None]
+    assert np.max(np.abs(err) - bound) <= 0, f"element error {np.max(np.abs(err) / bound):.3f} of the bound"
