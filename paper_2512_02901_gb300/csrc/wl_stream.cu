@@ -374,10 +374,12 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
       // Units past the first kSlots need MMAs, i.e. x: wait for the previous kernel first, so
       // that no bounded wait below counts its run time.
       if (l == kSlots) pdl_wait_primary();
-      if (l >= kSlots &&   // the slot's previous unit has been multiplied
-          !__all_sync(0xffffffffu, mbar_test_wait(&sfree[si], ph ^ 1u) ||
-                                       wait_or_abort(&sfree[si], ph ^ 1u, abort_flag, a.status)))
-        break;
+      if (l >= kSlots) {   // the slot's previous unit has been multiplied
+        if (!__all_sync(0xffffffffu, mbar_test_wait(&sfree[si], ph ^ 1u) ||
+                                         wait_or_abort(&sfree[si], ph ^ 1u, abort_flag, a.status)))
+          break;
+        tc_fence_after();   // the stores below follow the MMAs that read the slot
+      }
       const uint32_t a_col = t_lane + si * kSlotCols;
       uint32_t rr[32];
       if constexpr (kF4) {   // word w -> columns 4 w .. 4 w + 3
