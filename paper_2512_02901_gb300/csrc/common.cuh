@@ -3,6 +3,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 #include "fairy2i.h"
 
 namespace fairy2i {
@@ -49,4 +51,20 @@ inline fairy2i_status launch_status() {
 }
 // Per-device status word (defined in api.cu).
 unsigned int* device_status_word();
+
+// Raises the dynamic shared-memory limit of kernel `kern` to `bytes` on the current device, once
+// per device (function attributes belong to a device's context); `done` is the caller's mask of
+// devices already set (devices 0..63). Concurrent first calls set it twice, harmlessly.
+template <typename Kernel>
+inline bool smem_attr_once(Kernel kern, int bytes, std::atomic<uint64_t>& done) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
+  const uint64_t bit = uint64_t(1) << dev;
+  if (done.load(std::memory_order_acquire) & bit) return true;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes) !=
+      cudaSuccess)
+    return false;
+  done.fetch_or(bit, std::memory_order_release);
+  return true;
+}
 }  // namespace fairy2i

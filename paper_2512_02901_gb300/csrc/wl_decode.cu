@@ -398,13 +398,8 @@ inline Layout layout(int nchunks, int T, int NB) {
 template <int NB, int T>
 fairy2i_status launch(Args a, int count, const Layout& L, cudaStream_t stream) {
   auto kern = wl_decode_fp8_kernel<NB, T>;
-  static bool configured = false;
-  if (!configured) {
-    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem) !=
-        cudaSuccess)
-      return FAIRY2I_ERR_CUDA;
-    configured = true;
-  }
+  static std::atomic<uint64_t> smem_set{0};
+  if (!smem_attr_once(kern, kMaxSmem, smem_set)) return FAIRY2I_ERR_CUDA;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)(a.tiles * count));
   cfg.blockDim = dim3(kThreads);

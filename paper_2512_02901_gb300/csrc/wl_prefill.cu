@@ -425,13 +425,8 @@ template <int T>
 fairy2i_status launch(const Args& a, const CUtensorMap& xre, const CUtensorMap& xim, int grid,
                       cudaStream_t stream) {
   auto kern = wl_prefill_kernel<T>;
-  static bool configured = false;
-  if (!configured) {
-    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) !=
-        cudaSuccess)
-      return FAIRY2I_ERR_CUDA;
-    configured = true;
-  }
+  static std::atomic<uint64_t> smem_set{0};
+  if (!smem_attr_once(kern, kSmemBytes, smem_set)) return FAIRY2I_ERR_CUDA;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)grid);
   cfg.blockDim = dim3(kThreads);

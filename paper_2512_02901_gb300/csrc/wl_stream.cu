@@ -948,13 +948,8 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
 template <int NB, int T>
 fairy2i_status launch(const Args& a, int64_t grid, cudaStream_t stream) {
   auto kern = wl_stream_kernel<NB, T>;
-  static bool configured = false;
-  if (!configured) {
-    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             Layout<NB>::kSmemBytes) != cudaSuccess)
-      return FAIRY2I_ERR_CUDA;
-    configured = true;
-  }
+  static std::atomic<uint64_t> smem_set{0};
+  if (!smem_attr_once(kern, Layout<NB>::kSmemBytes, smem_set)) return FAIRY2I_ERR_CUDA;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)grid);
   cfg.blockDim = dim3(Layout<NB>::kThreads);

@@ -622,13 +622,8 @@ __global__ void __launch_bounds__(kThreads, 1) wl_tc_decode_kernel(const Args a)
 template <int NB, int T>
 fairy2i_status launch(const Args& a, int64_t grid, cudaStream_t stream) {
   auto kern = wl_tc_decode_kernel<NB, T>;
-  static bool configured = false;
-  if (!configured) {
-    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) !=
-        cudaSuccess)
-      return FAIRY2I_ERR_CUDA;
-    configured = true;
-  }
+  static std::atomic<uint64_t> smem_set{0};
+  if (!smem_attr_once(kern, kSmemBytes, smem_set)) return FAIRY2I_ERR_CUDA;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)grid);
   cfg.blockDim = dim3(kThreads);
