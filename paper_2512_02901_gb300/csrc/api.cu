@@ -1,6 +1,7 @@
 // C ABI of the library: argument validation, the per-device status word, dispatch.
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <mutex>
 
 #include "common.cuh"
@@ -70,12 +71,16 @@ static bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintp
 // several waves and the persistent tcgen05 kernel (one wave, every CTA looping over row blocks)
 // is faster; with at most one wave the warp-MMA kernel's shorter launch wins.
 static bool prefer_stream(int64_t n, int count) {
-  static int sms[64];
+  static std::atomic<int> sms[64];   // per device, 0 = not read yet
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
-  if (!sms[dev] && cudaDeviceGetAttribute(&sms[dev], cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
-    return false;
-  return (int64_t)count * ((n + 15) / 16) > sms[dev];
+  int v = sms[dev].load(std::memory_order_relaxed);
+  if (!v) {
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || v < 1)
+      return false;
+    sms[dev].store(v, std::memory_order_relaxed);
+  }
+  return (int64_t)count * ((n + 15) / 16) > v;
 }
 
 }  // namespace fairy2i
