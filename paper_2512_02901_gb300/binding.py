@@ -216,3 +216,17 @@ class Fairy2iLinear:
 
     def __call__(self, x: torch.Tensor, path: int = PATH_AUTO) -> torch.Tensor:
         return wl_matmul(x, self.codes, self.scales, self.out_features, path=path)
+
+    def save(self, path: str) -> None:
+        """Writes the packed codes and scales (see artifact.py for the format)."""
+        from . import artifact
+        artifact.save(path, self.codes, self.scales, self.out_features, self.in_features, self.T)
+
+    @classmethod
+    def load(cls, path: str, device="cuda") -> "Fairy2iLinear":
+        """A layer from a file written by save(), without the original weight."""
+        from . import artifact
+        layer = cls.__new__(cls)
+        layer.codes, layer.scales, layer.out_features, layer.in_features, layer.T = \
+            artifact.load(path, device)
+        return layer
