@@ -140,8 +140,14 @@ fairy2i_status fairy2i_quantize_noalloc(const float* U, const float* W, int64_t 
  *         m = ceil(in_features/2).
  *   codes, scales  as written by fairy2i_quantize for (n, m, T), n = ceil(out_features/2).
  *   y     float32 [B][ldy], overwritten: y[0:n] = Re y, y[n:out_features] = Im y.
- *   The result equals the float64 value of the sum up to float32 accumulation (the library
- *   picks a memory-bound decode kernel or a tensor-core kernel by B; both accumulate in fp32).
+ *   Accuracy: every kernel accumulates in fp32. The general (fp32 x) and prefill kernels use x
+ *   exactly; the decode kernels (bf16 x, B <= 2) hold each x entry in fixed point relative to
+ *   the largest |x| of the part of the K range one warp or CTA handles: the one-token
+ *   persistent kernel to half a unit of 2^-25 of it, the e4m3 kernels (warp-MMA, two-token
+ *   persistent, path 2) exactly down to ~2^-13 of it and to ~2^-22 below. Each output is then
+ *   within 1e-4 |x~|_1 sum_t max(s_re, s_im) (U and W terms) of the float64 value for any x on
+ *   the fp32, prefill and one-token persistent kernels, and on the e4m3 kernels unless hundreds
+ *   of entries of one part lie in (0, ~2^-13) of its maximum. Non-finite x: y unspecified.
  *   Requirements: B >= 0 (B = 0 is a no-op), in_features, out_features >= 1, 1 <= T <= 8,
  *   ldx >= in_features, ldy >= out_features, codes and x 16-byte aligned, y 4-byte aligned.
  * ------------------------------------------------------------------------------------------ */
