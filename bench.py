@@ -52,12 +52,10 @@ def peaks():
         return 6800.0, 1900.0, "fallback"
 
 
-# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) from ncu captures of the current
-# kernels (profiles/wl_decode_fp8_llama2_7b_stack_b1.md, profiles/wl_prefill_llama2_7b_2048tok.md):
-# one decoder layer's decode launches (every layer has the same shapes; grouped: q/k/v, o,
-# gate/up, down; ungrouped: seven), and one T = 2 prefill launch of the 4096 -> 11008 layer on
-# 2048 tokens.
-# Per call of a decoder layer and decode kernel: "fp8" = the warp-MMA kernel, "stream" = the
+# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) per launch, from ncu captures of the
+# current kernels: one decoder layer's decode launches (every layer has the same shapes; grouped:
+# q/k/v, o, gate/up, down; ungrouped: seven), and one T = 2 prefill launch of the 4096 -> 11008
+# layer on 2048 tokens. Per call and decode kernel: "fp8" = the warp-MMA kernel, "stream" = the
 # persistent tcgen05 kernel (grouped calls: q/k/v, gate/up).
 DECODE_DRAM_BYTES = {
     "fp8": {"q,k,v": 12.621e6, "o": 4.232e6, "gate,up": 22.582e6, "down": 11.323e6,

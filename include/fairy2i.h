@@ -121,6 +121,11 @@ fairy2i_status fairy2i_quantize(const float* U, const float* W, int64_t n, int64
  *    larger sizes return FAIRY2I_ERR_WORKSPACE and enqueue nothing.
  *  - The first call on a device looks up the array's device address (cudaGetSymbolAddress,
  *    with that device current); make that first call before any stream capture on the device.
+ *  - The array's 4 MiB are committed when the library's device code is loaded on a device. With
+ *    CUDA's lazy module loading (the default) that happens at the first call that needs it, and
+ *    it can then fail with FAIRY2I_ERR_CUDA if a host framework's pool already holds all device
+ *    memory: make the first call on each device before the framework reserves its pool (later
+ *    calls commit nothing).
  *  - All calls share the one array, on every stream: calls whose kernels overlap on the GPU
  *    (different streams without ordering between them) race and give wrong results. Calls
  *    ordered on one stream are safe; each call writes every scratch entry before reading it.
@@ -144,7 +149,7 @@ fairy2i_status fairy2i_quantize_noalloc(const float* U, const float* W, int64_t 
  *   exactly; the decode kernels (bf16 x, B <= 2) hold each x entry in fixed point relative to
  *   the largest |x| of the part of the K range one warp or CTA handles: the one-token
  *   persistent kernel to half a unit of 2^-25 of it, the e4m3 kernels (warp-MMA, two-token
- *   persistent, path 2) exactly down to ~2^-13 of it and to ~2^-22 below. Each output is then
+ *   persistent) exactly down to ~2^-13 of it and to ~2^-22 below. Each output is then
  *   within 1e-4 |x~|_1 sum_t max(s_re, s_im) (U and W terms) of the float64 value for any x on
  *   the fp32, prefill and one-token persistent kernels, and on the e4m3 kernels unless hundreds
  *   of entries of one part lie in (0, ~2^-13) of its maximum. Non-finite x: y unspecified.
@@ -161,9 +166,7 @@ fairy2i_status fairy2i_wl_matmul(const void* x, fairy2i_dtype xdt, int64_t B,
  *       (4) when the call's 16-row tiles outnumber the SMs, else the warp-MMA one (1); B > 2 ->
  *       the tcgen05 prefill GEMM where it applies (see 3); otherwise the general CUDA-core kernel;
  *   1 = the decode kernel where it applies, otherwise the general kernel;
- *   2 = the tcgen05 decode kernel (5th-generation tensor cores, the code matrix in tensor
- *       memory); it takes B <= 2 bf16 tokens, T <= 4 and rows of at most 176 128-code chunks
- *       (in_features <= 45056) and returns FAIRY2I_ERR_INVALID_ARG for anything else;
+ *   2 = retired (an earlier tcgen05 decode kernel); returns FAIRY2I_ERR_INVALID_ARG;
  *   3 = the tcgen05 prefill GEMM (codes expanded into bf16 +-1 tiles in tensor memory, x by TMA,
  *       64 tokens per tile); it takes bf16 x with 16-byte aligned rows, ldx % 8 == 0,
  *       m % 8 == 0 (m = ceil(in_features/2)) and T <= 4, and returns FAIRY2I_ERR_INVALID_ARG for
@@ -175,7 +178,7 @@ fairy2i_status fairy2i_wl_matmul(const void* x, fairy2i_dtype xdt, int64_t B,
  *       which keeps every output within the per-element bound for any x; two tokens: e4m3
  *       operands, x as two e4m3 limbs); it takes B <= 2 bf16 tokens, T <= 4 and
  *       in_features <= 24576 and returns FAIRY2I_ERR_INVALID_ARG for anything else.
- * The decode kernels (paths 1, 2, 4) read the codes and scales before waiting for the previous
+ * The decode kernels (paths 1, 4) read the codes and scales before waiting for the previous
  * kernel in the stream (programmatic dependent launch): the codes must not be written by the
  * kernel launched right before the matmul on the same stream unless that kernel is one of this
  * library's convert/quantize/adjoint kernels, which end before any dependent kernel starts.

@@ -14,7 +14,7 @@ Two arithmetic modes
 ``math``      plain float64 everywhere, no float32 rounding, scales kept as exact float64
               quotients. Used for the mathematical pins (Theorem 1, the residual-norm identity).
 
-Readings where the paper is silent (each also listed in the design doc):
+Readings where the paper is silent:
 * real/imaginary pairing of a real vector is by halves: x~ = [Re x ; Im x]  (Sec. 3.1);
 * an odd real dimension is padded by one zero channel appended at its end (Sec. 3.1, Remarks);
 * ties of the phase projection are broken the way k = floor(2*theta/pi + 1/2) breaks them, and

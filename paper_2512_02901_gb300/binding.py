@@ -12,7 +12,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libfairy2i.so")
 
 F32, BF16 = 0, 1
-PATH_AUTO, PATH_DECODE, PATH_TC_DECODE, PATH_TC_PREFILL, PATH_STREAM = 0, 1, 2, 3, 4
+PATH_AUTO, PATH_DECODE, PATH_TC_PREFILL, PATH_STREAM = 0, 1, 3, 4
 MAX_STAGES = 8
 STATUS = {0: "ok", 1: "invalid argument", 2: "shape", 3: "alignment", 4: "dtype", 5: "workspace",
           6: "non-finite weight", 7: "device wait timeout", 8: "CUDA error"}
@@ -127,6 +127,30 @@ def quantize(U: torch.Tensor, W: torch.Tensor, T: int, codes=None, scales=None, 
     return codes, scales
 
 
+def check_layer(codes: torch.Tensor, scales: torch.Tensor, out_features: int, in_features: int,
+                T: int, device=None) -> None:
+    """Raises ValueError unless (codes, scales) can hold a T-stage layer of out_features x
+    in_features on `device`: the packed words at least fairy2i_codes_words(n, m, T) (int32 or
+    uint32, contiguous) and float32 contiguous scales of at least [T][2][2]. A mismatch would let
+    a kernel read past the end of the codes buffer, so it is caught before any launch."""
+    if not (1 <= T <= MAX_STAGES):
+        raise ValueError(f"T = {T} outside 1..{MAX_STAGES}")
+    if out_features < 1 or in_features < 1:
+        raise ValueError("out_features and in_features must be >= 1")
+    n, m = complex_dims(out_features, in_features)
+    need = T * 2 * ((n + 15) // 16) * 16 * (((m + 127) // 128) * 8)
+    if codes.dtype not in (torch.int32, torch.uint32) or not codes.is_contiguous():
+        raise ValueError("codes must be a contiguous int32/uint32 tensor of packed words")
+    if codes.numel() < need:
+        raise ValueError(f"codes hold {codes.numel()} words, a {T}-stage {out_features}x"
+                         f"{in_features} layer needs {need}")
+    if scales.dtype != torch.float32 or not scales.is_contiguous() or scales.numel() < 4 * T:
+        raise ValueError(f"scales must be contiguous float32 with at least [T][2][2] = {4 * T} "
+                         f"values (got {tuple(scales.shape)}, {scales.dtype})")
+    if device is not None and (codes.device != device or scales.device != device):
+        raise ValueError(f"codes ({codes.device}) and scales ({scales.device}) must be on {device}")
+
+
 def wl_matmul(x: torch.Tensor, codes: torch.Tensor, scales: torch.Tensor, out_features: int,
               y=None, path: int = PATH_AUTO, stream=None, T: int | None = None):
     """x [B][in_features] float32/bf16 -> y float32 [B][out_features] = [Re y | Im y].
@@ -143,8 +167,11 @@ def wl_matmul(x: torch.Tensor, codes: torch.Tensor, scales: torch.Tensor, out_fe
     B, in_features = x.shape
     if T is None:
         T = scales.shape[0]
+    check_layer(codes, scales, out_features, in_features, T, x.device)
     if y is None:
         y = torch.empty((B, out_features), dtype=torch.float32, device=x.device)
+    assert y.is_cuda and y.dtype == torch.float32 and y.stride(1) == 1 and \
+        y.shape[0] >= B and y.shape[1] >= out_features
     xdt = F32 if x.dtype == torch.float32 else BF16
     _check("fairy2i_wl_matmul",
            load().fairy2i_wl_matmul_path(_ptr(x), xdt, B, in_features, x.stride(0), _ptr(codes),
@@ -165,10 +192,14 @@ def wl_matmul_group(x: torch.Tensor, codes, scales, out_features: int, ys=None, 
     B, in_features = x.shape
     if T is None:
         T = scales[0].shape[0]
+    for c, s in zip(codes, scales):
+        check_layer(c, s, out_features, in_features, T, x.device)
     if ys is None:
         ys = [torch.empty((B, out_features), dtype=torch.float32, device=x.device)
               for _ in range(count)]
     assert len(ys) == count and all(y.stride(0) == ys[0].stride(0) for y in ys)
+    assert all(y.is_cuda and y.dtype == torch.float32 and y.stride(1) == 1 and
+               y.shape[0] >= B and y.shape[1] >= out_features for y in ys)
     arr = ctypes.c_void_p * count
     cp = arr(*[c.data_ptr() for c in codes])
     sp = arr(*[s.data_ptr() for s in scales])

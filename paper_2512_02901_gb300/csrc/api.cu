@@ -22,10 +22,6 @@ fairy2i_status launch_wl_decode(const void* x, fairy2i_dtype xdt, int64_t B, int
                                 int64_t ldx, const uint32_t* codes, const float* scales,
                                 int64_t n, int64_t m, int64_t out_features, int64_t wpr, int T,
                                 float* y, int64_t ldy, cudaStream_t stream, bool* handled);
-fairy2i_status launch_wl_tc(const void* x, fairy2i_dtype xdt, int64_t B, int64_t in_features,
-                            int64_t ldx, const uint32_t* codes, const float* scales, int64_t n,
-                            int64_t m, int64_t out_features, int64_t wpr, int T, float* y,
-                            int64_t ldy, cudaStream_t stream, bool* handled);
 fairy2i_status launch_wl_prefill(const void* x, fairy2i_dtype xdt, int64_t B, int64_t in_features,
                                  int64_t ldx, const uint32_t* codes, const float* scales,
                                  int64_t n, int64_t m, int64_t out_features, int64_t wpr, int T,
@@ -170,12 +166,7 @@ fairy2i_status fairy2i_wl_matmul_path(const void* x, fairy2i_dtype xdt, int64_t 
     if (handled || st != FAIRY2I_OK) return st;
     return FAIRY2I_ERR_INVALID_ARG;   // shape or dtype outside the kernel
   }
-  if (path == 2) {   // tcgen05 decode kernel (explicit): B <= 2 bf16 tokens, T <= 4
-    st = launch_wl_tc(x, xdt, B, in_features, ldx, codes, scales, n, m, out_features, wpr, T, y,
-                      ldy, s, &handled);
-    if (handled || st != FAIRY2I_OK) return st;
-    return FAIRY2I_ERR_INVALID_ARG;   // shape or dtype outside the tcgen05 decode kernel
-  }
+  if (path == 2) return FAIRY2I_ERR_INVALID_ARG;   // retired
   if (path == 0 && B <= 2 && xdt == FAIRY2I_BF16 && prefer_stream(n, 1)) {
     st = launch_wl_stream_group(x, xdt, B, in_features, ldx, 1, &codes, &scales, n, m,
                                 out_features, wpr, T, &y, ldy, s, &handled);

@@ -274,66 +274,21 @@ def test_wl_decode_all_codes_each_value(F):
     assert_wl_close(yg, O.wl_matmul(xo, codes, scales, 2 * n), xo, scales)
 
 
-# ------------------------------------------------------------------------------ tcgen05 decode
-@pytest.mark.parametrize("out_f,in_f,T,B", [
-    (32, 32, 1, 1), (31, 515, 2, 2), (64, 256, 3, 1), (4096, 4096, 4, 1), (100, 8192, 3, 2),
-    (17, 2, 2, 1), (4096, 11008, 2, 2), (11008, 4096, 2, 1), (48, 1024, 2, 2),
-    (4096, 4096, 2, 1), (130, 45056, 2, 1),
-])
-def test_wl_tcgen05_decode_path(F, out_f, in_f, T, B):
-    """The tcgen05 decode kernel (path 2) on ragged rows and chunks, every T it takes, clusters of
-    1..8 CTAs per row block (in_features 45056: 176 chunks, 8 CTAs of 22), odd in_features (x
-    staged by plain loads) and 16-byte-aligned rows (x staged by bulk copy)."""
-    n, m = O.complex_dims(out_f, in_f)
-    codes, scales = _random_quantized(n, m, T, seed=3 * out_f + 5 * in_f + T)
-    x = synth.outlier_activations(B, in_f, seed=out_f + in_f + 1)
-    yg = _run_wl(F, x, codes, scales, out_f, path=2)
-    xo = x.float().numpy()
-    assert_wl_close(yg, O.wl_matmul(xo, codes, scales, out_f), xo, scales)
-
-
-@pytest.mark.parametrize("T", [1, 2, 3, 4])
-def test_wl_tcgen05_all_codes_each_value(F, T):
-    """Every code value at every word position of every stage-matrix lane block."""
-    n, m = 40, 384
-    codes = np.zeros((T, 2, n, m), dtype=np.uint8)
-    for t in range(T):
-        for j in range(n):
-            codes[t, 0, j] = (np.arange(m) + j + t) % 4
-            codes[t, 1, j] = (np.arange(m) // 16 + 3 * j + t) % 4
-    g = np.random.default_rng(T)
-    scales = (0.01 + 0.02 * g.random((T, 2, 2))).astype(np.float32)
-    x = synth.outlier_activations(2, 2 * m, seed=7 + T)
-    yg = _run_wl(F, x, codes, scales, 2 * n, path=2)
-    xo = x.float().numpy()
-    assert_wl_close(yg, O.wl_matmul(xo, codes, scales, 2 * n), xo, scales)
-
-
-def test_wl_tcgen05_strided_x_and_y(F):
-    n, m, T, B = 70, 136, 2, 2
-    codes, scales = _random_quantized(n, m, T, seed=11)
-    xbig = synth.outlier_activations(B, 2 * m + 24, seed=12)
-    x = xbig.to(DEV)[:, : 2 * m]
-    y = torch.full((B, 2 * n + 8), 7.0, device=DEV)
-    F.wl_matmul(x, upload_codes(O.pack_codes(codes)), torch.from_numpy(scales).to(DEV), 2 * n,
-                y=y[:, : 2 * n], path=2)
-    assert F.get_status() == 0
-    yg = y.cpu().numpy()
-    assert np.all(yg[:, 2 * n:] == 7.0)
-    xo = xbig[:, : 2 * m].float().numpy()
-    assert_wl_close(yg[:, : 2 * n], O.wl_matmul(xo, codes, scales, 2 * n), xo, scales)
-
-
-def test_wl_tcgen05_rejects_outside_its_domain(F):
+# ------------------------------------------------------------------------------ retired path 2
+def test_retired_path_2_is_rejected(F):
+    """Path 2 (an earlier tcgen05 decode kernel, slower than both decode kernels that replaced
+    it) is retired: every call naming it returns FAIRY2I_ERR_INVALID_ARG and enqueues nothing."""
     n, m, T = 16, 64, 2
     codes, scales = _random_quantized(n, m, T, seed=13)
     cd = upload_codes(O.pack_codes(codes))
     sc = torch.from_numpy(scales).to(DEV)
-    for x in (synth.outlier_activations(3, 2 * m, seed=1).to(DEV),          # B = 3
-              torch.zeros((1, 2 * m), dtype=torch.float32, device=DEV)):    # fp32 x
+    for x in (synth.outlier_activations(1, 2 * m, seed=1).to(DEV),
+              synth.outlier_activations(3, 2 * m, seed=1).to(DEV),
+              torch.zeros((1, 2 * m), dtype=torch.float32, device=DEV)):
         with pytest.raises(F.Fairy2iError) as e:
             F.wl_matmul(x, cd, sc, 2 * n, path=2)
         assert e.value.code == 1
+    assert F.get_status() == 0
 
 
 # ------------------------------------------------------------------------------ tcgen05 prefill
@@ -504,3 +459,32 @@ def test_input_gradient_through_adjoint_codes(F, out_f, in_f, T, B, dtype):
     go = gy.float().numpy()
     want = O.wl_matmul(go, O.adjoint_codes(codes), scales, in_f)
     assert_wl_close(gx.cpu().numpy(), want, go, scales)
+
+
+# ------------------------------------------------------------------------------ stream ordering
+@pytest.mark.parametrize("path", [1, 4])
+def test_quantize_then_decode_back_to_back(F, path):
+    """The decode kernels read the codes and scales before their programmatic-launch wait. They
+    rely on the quantize kernel that wrote them (launched just before on the same stream, no
+    synchronization between) having ended first. Codes and scales start as garbage and each
+    round rewrites them, so a decode that read them early would differ from the oracle."""
+    out_f, in_f, T = 4096, 4096, 2
+    R = synth.student_t_weight(out_f, in_f, seed=91)
+    n, m = O.complex_dims(out_f, in_f)
+    Uo, Wo = O.convert(R.numpy())
+    co, so = O.quantize(Uo, Wo, T)
+    xs = [synth.outlier_activations(1, in_f, seed=92 + i) for i in range(3)]
+    Rd = R.to(DEV)
+    stream = torch.cuda.Stream()
+    with torch.cuda.stream(stream):
+        for x in xs:
+            codes = torch.full((T, 2, (n + 15) // 16, F.words_per_row(m) // 8, 16, 8), -1,
+                               dtype=torch.int32, device=DEV)
+            scales = torch.full((T, 2, 2), float("nan"), device=DEV)
+            U, W = F.convert(Rd, stream=stream)
+            F.quantize(U, W, T, codes=codes, scales=scales, stream=stream)
+            y = F.wl_matmul(x.to(DEV), codes, scales, out_f, path=path, stream=stream)
+            stream.synchronize()
+            xo = x.float().numpy()
+            assert_wl_close(y.cpu().numpy(), O.wl_matmul(xo, co, so, out_f), xo, so)
+    assert F.get_status(stream) == 0

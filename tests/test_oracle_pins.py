@@ -331,6 +331,49 @@ def test_wl_matmul_plus_i_uses_s_im():
     assert np.allclose(y[:, :n], expect.real[:, None]) and np.allclose(y[:, n:], expect.imag[:, None])
 
 
+def test_dequant_each_codeword_by_hand():
+    """Eq. ifairy-dequant with hand-written codewords i^c: c = 0 -> +1, 1 -> +i, 2 -> -1,
+    3 -> -i, the real part scaled by s_re and the imaginary part by s_im (s_re != s_im, so a
+    swapped scale or a wrong sign on any codeword fails)."""
+    s_re, s_im = np.float32(0.375), np.float32(2.5)
+    got = O.dequant(np.array([0, 1, 2, 3]), s_re, s_im)
+    want = np.array([0.375 + 0j, 2.5j, -0.375 + 0j, -2.5j])
+    assert np.array_equal(got, want)
+
+
+@pytest.mark.parametrize("shape", [(9, 14), (1, 1), (32, 5)])
+def test_dequant_is_the_residual_step(shape):
+    """R^(t) - dequant(B^(t), s^(t)) = R^(t+1) exactly (math mode): dequant agrees with the
+    residual update of Sec. 3.3, whose scales are pinned by the norm identity above."""
+    M = rng.standard_normal(shape) + 1j * rng.standard_normal(shape)
+    codes, scales, res = O.residual_quantize(M, 3, mode="math")
+    for t in range(3):
+        r = res[t][0] + 1j * res[t][1]
+        nxt = res[t + 1][0] + 1j * res[t + 1][1]
+        assert np.array_equal(r - O.dequant(codes[t], scales[t][0], scales[t][1]), nxt)
+
+
+@pytest.mark.parametrize("mat,code", [(0, 2), (0, 3), (1, 2), (1, 3)])
+def test_wl_matmul_minus_codes_closed_form(mat, code):
+    """All codes -1 (c = 2) or -i (c = 3) on one matrix, a large scale on the unused axis that
+    must not appear: U with -1 gives y = -s_re sum x, U with -i gives y = -i s_im sum x; on W the
+    same with conj(x) (Eq. widely-linear)."""
+    n, m = 4, 7
+    codes = np.zeros((1, 2, n, m), dtype=np.uint8)
+    codes[0, mat] = code
+    scales = np.zeros((1, 2, 2), dtype=np.float32)
+    s_used, s_unused = 0.625, 1000.0
+    scales[0, mat] = (s_used, s_unused) if code == 2 else (s_unused, s_used)
+    x = rng.standard_normal((2, 2 * m))
+    z = x[:, :m] + 1j * x[:, m:]
+    zz = z if mat == 0 else np.conj(z)
+    factor = -s_used if code == 2 else -1j * s_used
+    expect = factor * zz.sum(axis=1)
+    y = O.wl_matmul(x, codes, scales, 2 * n)
+    assert np.allclose(y[:, :n], expect.real[:, None], atol=1e-12)
+    assert np.allclose(y[:, n:], expect.imag[:, None], atol=1e-12)
+
+
 def test_unquantized_limit_is_theorem1():
     """Replacing the dequantized matrices by U, W reproduces R x~."""
     R = rng.standard_normal((10, 14))
