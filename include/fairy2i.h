@@ -177,7 +177,10 @@ fairy2i_status fairy2i_wl_matmul(const void* x, fairy2i_dtype xdt, int64_t B,
  *       operands, each x entry held to 2^-26 of the largest |x| in a CTA's part of the K range,
  *       which keeps every output within the per-element bound for any x; two tokens: e4m3
  *       operands, x as two e4m3 limbs); it takes B <= 2 bf16 tokens, T <= 4 and
- *       in_features <= 24576 and returns FAIRY2I_ERR_INVALID_ARG for anything else.
+ *       in_features <= 24576 and returns FAIRY2I_ERR_INVALID_ARG for anything else;
+ *   5 = the chained decode kernel (fairy2i_wl_matmul_chain) on this one call; it takes B = 1
+ *       token (float32 or bf16), T <= 4 and in_features <= 24576 and returns
+ *       FAIRY2I_ERR_INVALID_ARG for anything else.
  * The decode kernels (paths 1, 4) read the codes and scales before waiting for the previous
  * kernel in the stream (programmatic dependent launch): the codes must not be written by the
  * kernel launched right before the matmul on the same stream unless that kernel is one of this
@@ -230,7 +233,9 @@ fairy2i_status fairy2i_wl_matmul_group(const void* x, fairy2i_dtype xdt, int64_t
 /* fairy2i_wl_matmul_group with the decode kernel chosen by `path`: 0 = automatic (as above),
  * 1 = the warp-MMA decode kernel where it applies (else the automatic path per member),
  * 4 = the persistent tcgen05 decode kernel, one launch for the group (B <= 2 bf16 tokens, T <= 4,
- * in_features <= 24576; FAIRY2I_ERR_INVALID_ARG for anything else). Any other path returns
+ * in_features <= 24576; FAIRY2I_ERR_INVALID_ARG for anything else), 5 = the chained decode kernel
+ * on this one group (B = 1, T <= 4, in_features <= 24576; FAIRY2I_ERR_INVALID_ARG otherwise).
+ * Any other path returns
  * FAIRY2I_ERR_INVALID_ARG. Results agree with the separate calls within the float32-accumulation
  * tolerance (bit-identical for path 1). */
 fairy2i_status fairy2i_wl_matmul_group_path(const void* x, fairy2i_dtype xdt, int64_t B,
@@ -239,6 +244,56 @@ fairy2i_status fairy2i_wl_matmul_group_path(const void* x, fairy2i_dtype xdt, in
                                             const float* const* scales, int64_t out_features,
                                             int T, float* const* y, int64_t ldy, int path,
                                             void* stream);
+
+/* ------------------------------------------------------------------------------------------
+ * A chain of one-token calls in one launch: the linears of a decoder applied in data-flow
+ * order, e.g. per decoder layer q/k/v (one call of three linears on one input), o, gate/up, down
+ * (Eq. widely-linear with Eq. res-sum for every linear; Algorithm 1 with the scales of Eq.
+ * ifairy-dequant and the W conj(x) term).
+ *   Call c computes, for g < count, y[g] = fairy2i_wl_matmul(x, xdt, 1, in_features,
+ *   in_features, codes[g], scales[g], out_features, T, y[g], out_features), and reads x only
+ *   after every y of call c - 1 has been written: x of call c may be (a view of) a y of call
+ *   c - 1 when xdt is FAIRY2I_F32. The packed codes do not depend on the data and are streamed
+ *   ahead across calls.
+ *   calls        host array of ncalls descriptors (read before the call returns), 1 <= ncalls.
+ *                Chains longer than fairy2i_wl_matmul_chain_max_calls() run as several
+ *                launches, one after the other on `stream`.
+ *     x          one token: in_features entries of dtype xdt, [Re x | Im x], 16-byte aligned.
+ *     codes, scales  as written by fairy2i_quantize for (n, m, T) of that call's shape.
+ *     y          out_features float32 values [Re y | Im y] per linear, 4-byte aligned,
+ *                overwritten. The y of a call must not overlap its own x or codes, nor another
+ *                call's x, y or codes except as the x of the next call.
+ *   T            stages, the same for every call, 1 <= T <= 4.
+ *   cluster_size 0 picks the K split of the launch; 1, 2, 4 or 8 forces it (thread-block
+ *                clusters of that many CTAs split every row; every call then needs
+ *                ceil(in_features / 256) >= cluster_size and at most 24 cluster_size
+ *                128-code chunks per row).
+ *   workspace    >= fairy2i_wl_matmul_chain_workspace_bytes(ncalls) bytes of device memory,
+ *                16-byte aligned (completion counters, zeroed by the call on `stream`); may be
+ *                NULL when that size is 0 (one call).
+ *   Limits: in_features <= 24576 per call (FAIRY2I_ERR_INVALID_ARG otherwise, nothing enqueued).
+ *   Accuracy: x is held in fixed point, each entry to 2^-28 of the largest |x| in the part of
+ *   the K range one CTA handles; every output is within 1e-4 |x~|_1 sum_t max(s_re, s_im) (U and
+ *   W terms) of the float64 value for any x with in_features <= 24576.
+ *   The launch keeps one CTA on each SM it uses and its CTAs wait for one another between calls
+ *   (bounded: FAIRY2I_ERR_TIMEOUT in the status word after about a second), so a chain should
+ *   not share the device with other work that could hold SMs for that long.
+ * ------------------------------------------------------------------------------------------ */
+typedef struct {
+  const void* x;
+  fairy2i_dtype xdt;
+  int32_t count;                               /* linears sharing x, 1..FAIRY2I_MAX_GROUP */
+  int64_t in_features, out_features;
+  const uint32_t* codes[FAIRY2I_MAX_GROUP];
+  const float* scales[FAIRY2I_MAX_GROUP];
+  float* y[FAIRY2I_MAX_GROUP];
+} fairy2i_chain_call;
+
+int fairy2i_wl_matmul_chain_max_calls(void);
+size_t fairy2i_wl_matmul_chain_workspace_bytes(int ncalls);
+fairy2i_status fairy2i_wl_matmul_chain(const fairy2i_chain_call* calls, int ncalls, int T,
+                                       int cluster_size, void* workspace, size_t workspace_bytes,
+                                       void* stream);
 
 /* ------------------------------------------------------------------------------------------
  * Synchronizes `stream`, then returns and clears the device-side status of the current

@@ -12,7 +12,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libfairy2i.so")
 
 F32, BF16 = 0, 1
-PATH_AUTO, PATH_DECODE, PATH_TC_PREFILL, PATH_STREAM = 0, 1, 3, 4
+PATH_AUTO, PATH_DECODE, PATH_TC_PREFILL, PATH_STREAM, PATH_CHAIN = 0, 1, 3, 4, 5
 MAX_STAGES = 8
 STATUS = {0: "ok", 1: "invalid argument", 2: "shape", 3: "alignment", 4: "dtype", 5: "workspace",
           6: "non-finite weight", 7: "device wait timeout", 8: "CUDA error"}
@@ -42,6 +42,20 @@ SIGNATURES = {
                                       _vp, _i64, _int, _vp], _int),
 }
 MAX_GROUP = 4
+
+
+class ChainCall(ctypes.Structure):
+    """fairy2i_chain_call: one call of a chained decode (one token, up to MAX_GROUP linears)."""
+    _fields_ = [("x", _vp), ("xdt", _int), ("count", ctypes.c_int32),
+                ("in_features", _i64), ("out_features", _i64),
+                ("codes", _vp * 4), ("scales", _vp * 4), ("y", _vp * 4)]
+
+
+SIGNATURES.update({
+    "fairy2i_wl_matmul_chain_max_calls": ([], _int),
+    "fairy2i_wl_matmul_chain_workspace_bytes": ([_int], _sz),
+    "fairy2i_wl_matmul_chain": ([_vp, _int, _int, _int, _vp, _sz, _vp], _int),
+})
 
 
 class Fairy2iError(RuntimeError):
@@ -211,6 +225,60 @@ def wl_matmul_group(x: torch.Tensor, codes, scales, out_features: int, ys=None, 
                                                out_features, T, ctypes.cast(yp, _vp),
                                                ys[0].stride(0), path, _stream(stream)))
     return ys
+
+
+def chain_workspace(ncalls: int, device) -> torch.Tensor:
+    """Device workspace (completion counters) for a chain of ncalls calls."""
+    nbytes = int(load().fairy2i_wl_matmul_chain_workspace_bytes(ncalls))
+    return torch.empty(max(nbytes, 16), dtype=torch.uint8, device=device)
+
+
+def chain_calls(calls):
+    """ctypes array of fairy2i_chain_call from (x, codes list, scales list, y list, out_features)
+    tuples; x is one token [1][in_features] (float32 or bf16, CUDA), y [1][out_features] float32.
+    The layers are checked like wl_matmul's."""
+    arr = (ChainCall * len(calls))()
+    T = None
+    for i, (x, codes, scales, ys, out_features) in enumerate(calls):
+        assert x.is_cuda and x.dim() == 2 and x.shape[0] == 1 and x.is_contiguous()
+        assert x.dtype in (torch.float32, torch.bfloat16)
+        count = len(codes)
+        assert count == len(scales) == len(ys) and 1 <= count <= MAX_GROUP
+        in_features = x.shape[1]
+        if T is None:
+            T = scales[0].shape[0]
+        for c, s, y in zip(codes, scales, ys):
+            check_layer(c, s, out_features, in_features, T, x.device)
+            assert y.is_cuda and y.dtype == torch.float32 and y.is_contiguous() and \
+                y.numel() >= out_features
+        k = arr[i]
+        k.x = x.data_ptr()
+        k.xdt = F32 if x.dtype == torch.float32 else BF16
+        k.count = count
+        k.in_features, k.out_features = in_features, out_features
+        for g in range(count):
+            k.codes[g] = codes[g].data_ptr()
+            k.scales[g] = scales[g].data_ptr()
+            k.y[g] = ys[g].data_ptr()
+    return arr
+
+
+def wl_matmul_chain(calls, T: int, cluster_size: int = 0, workspace=None, stream=None,
+                    arr=None):
+    """Runs a chain of one-token calls in one launch (fairy2i_wl_matmul_chain): call c reads its
+    x only after every y of call c - 1 is written. `calls`: (x, codes, scales, ys, out_features)
+    tuples (see chain_calls), or None with `arr` a prepared chain_calls() array."""
+    if arr is None:
+        arr = chain_calls(calls)
+    n = len(arr)
+    if workspace is None:
+        dev = torch.device("cuda", torch.cuda.current_device()) if calls is None else \
+            calls[0][0].device
+        workspace = chain_workspace(n, dev)
+    _check("fairy2i_wl_matmul_chain",
+           load().fairy2i_wl_matmul_chain(ctypes.cast(arr, _vp), n, T, cluster_size,
+                                          _ptr(workspace), workspace.numel(), _stream(stream)))
+    return arr
 
 
 def codes_adjoint(codes: torch.Tensor, n: int, m: int, T: int, stream=None) -> torch.Tensor:

@@ -33,6 +33,9 @@ fairy2i_status launch_wl_stream_group(const void* x, fairy2i_dtype xdt, int64_t 
                                       int T, float* const* y, int64_t ldy, cudaStream_t stream,
                                       bool* handled);
 fairy2i_status launch_selftest_wait(uint32_t limit_us, cudaStream_t stream);
+fairy2i_status launch_wl_chain(const fairy2i_chain_call* calls, int ncalls, int T,
+                               int cluster_size, unsigned int* done, cudaStream_t stream);
+int chain_max_calls();
 fairy2i_status launch_codes_adjoint(const uint32_t* codes, int64_t n, int64_t m, int T,
                                     uint32_t* codes_adj, cudaStream_t stream);
 fairy2i_status launch_wl_decode_group(const void* x, fairy2i_dtype xdt, int64_t B,
@@ -141,7 +144,7 @@ fairy2i_status fairy2i_wl_matmul_path(const void* x, fairy2i_dtype xdt, int64_t 
                                       const float* scales, int64_t out_features, int T, float* y,
                                       int64_t ldy, int path, void* stream) {
   if (B < 0 || in_features < 1 || out_features < 1 || T < 1 || T > FAIRY2I_MAX_STAGES ||
-      path < 0 || path > 4)
+      path < 0 || path > 5)
     return FAIRY2I_ERR_INVALID_ARG;
   if (xdt != FAIRY2I_F32 && xdt != FAIRY2I_BF16) return FAIRY2I_ERR_DTYPE;
   if (B == 0) return FAIRY2I_OK;
@@ -167,6 +170,19 @@ fairy2i_status fairy2i_wl_matmul_path(const void* x, fairy2i_dtype xdt, int64_t 
     return FAIRY2I_ERR_INVALID_ARG;   // shape or dtype outside the kernel
   }
   if (path == 2) return FAIRY2I_ERR_INVALID_ARG;   // retired
+  if (path == 5) {   // the chained decode kernel on this one call
+    if (B != 1 || ldy < out_features) return FAIRY2I_ERR_INVALID_ARG;
+    fairy2i_chain_call c = {};
+    c.x = x;
+    c.xdt = xdt;
+    c.count = 1;
+    c.in_features = in_features;
+    c.out_features = out_features;
+    c.codes[0] = codes;
+    c.scales[0] = scales;
+    c.y[0] = y;
+    return fairy2i_wl_matmul_chain(&c, 1, T, 0, nullptr, 0, stream);
+  }
   if (path == 0 && B <= 2 && xdt == FAIRY2I_BF16 && prefer_stream(n, 1)) {
     st = launch_wl_stream_group(x, xdt, B, in_features, ldx, 1, &codes, &scales, n, m,
                                 out_features, wpr, T, &y, ldy, s, &handled);
@@ -194,7 +210,7 @@ fairy2i_status fairy2i_wl_matmul_group_path(const void* x, fairy2i_dtype xdt, in
                                             int T, float* const* y, int64_t ldy, int path,
                                             void* stream) {
   if (count < 1 || count > FAIRY2I_MAX_GROUP || !codes || !scales || !y ||
-      (path != 0 && path != 1 && path != 4))
+      (path != 0 && path != 1 && path != 4 && path != 5))
     return FAIRY2I_ERR_INVALID_ARG;
   // Every member is validated as a single call would be (B = 0 included) before anything runs.
   for (int g = 0; g < count; ++g) {
@@ -206,6 +222,21 @@ fairy2i_status fairy2i_wl_matmul_group_path(const void* x, fairy2i_dtype xdt, in
     if (ldx < in_features || ldy < out_features) return FAIRY2I_ERR_SHAPE;
     if (!aligned(x, 16) || !aligned(codes[g], 16) || !aligned(y[g], 4) || !aligned(scales[g], 4))
       return FAIRY2I_ERR_ALIGNMENT;
+  }
+  if (path == 5) {   // the chained decode kernel on this one group
+    if (B != 1) return FAIRY2I_ERR_INVALID_ARG;
+    fairy2i_chain_call c = {};
+    c.x = x;
+    c.xdt = xdt;
+    c.count = count;
+    c.in_features = in_features;
+    c.out_features = out_features;
+    for (int g = 0; g < count; ++g) {
+      c.codes[g] = codes[g];
+      c.scales[g] = scales[g];
+      c.y[g] = y[g];
+    }
+    return fairy2i_wl_matmul_chain(&c, 1, T, 0, nullptr, 0, stream);
   }
   const int64_t n = (out_features + 1) / 2, m = (in_features + 1) / 2;
   const int64_t wpr = fairy2i_codes_words_per_row(m);
@@ -241,6 +272,57 @@ fairy2i_status fairy2i_wl_matmul_group(const void* x, fairy2i_dtype xdt, int64_t
                                        void* stream) {
   return fairy2i_wl_matmul_group_path(x, xdt, B, in_features, ldx, count, codes, scales,
                                       out_features, T, y, ldy, 0, stream);
+}
+
+int fairy2i_wl_matmul_chain_max_calls(void) { return chain_max_calls(); }
+
+size_t fairy2i_wl_matmul_chain_workspace_bytes(int ncalls) {
+  if (ncalls <= 1) return 0;
+  const int per = chain_max_calls();
+  const int counters = ncalls < per ? ncalls : per;
+  return ((size_t)counters * sizeof(unsigned int) + 255) & ~(size_t)255;
+}
+
+fairy2i_status fairy2i_wl_matmul_chain(const fairy2i_chain_call* calls, int ncalls, int T,
+                                       int cluster_size, void* workspace, size_t workspace_bytes,
+                                       void* stream) {
+  if (!calls || ncalls < 1 || T < 1 || T > 4) return FAIRY2I_ERR_INVALID_ARG;
+  if (cluster_size != 0 && cluster_size != 1 && cluster_size != 2 && cluster_size != 4 &&
+      cluster_size != 8)
+    return FAIRY2I_ERR_INVALID_ARG;
+  // Every call is validated before anything is enqueued.
+  for (int c = 0; c < ncalls; ++c) {
+    const fairy2i_chain_call& k = calls[c];
+    if (k.count < 1 || k.count > FAIRY2I_MAX_GROUP || k.in_features < 1 || k.out_features < 1 ||
+        !k.x)
+      return FAIRY2I_ERR_INVALID_ARG;
+    if (k.xdt != FAIRY2I_F32 && k.xdt != FAIRY2I_BF16) return FAIRY2I_ERR_DTYPE;
+    if (k.in_features > 24576 || k.out_features > (int64_t(1) << 30))
+      return FAIRY2I_ERR_INVALID_ARG;
+    if (!aligned(k.x, 16)) return FAIRY2I_ERR_ALIGNMENT;
+    for (int g = 0; g < k.count; ++g) {
+      if (!k.codes[g] || !k.scales[g] || !k.y[g]) return FAIRY2I_ERR_INVALID_ARG;
+      if (!aligned(k.codes[g], 16) || !aligned(k.scales[g], 4) || !aligned(k.y[g], 4))
+        return FAIRY2I_ERR_ALIGNMENT;
+    }
+  }
+  const size_t need = fairy2i_wl_matmul_chain_workspace_bytes(ncalls);
+  if (need > 0 && (!workspace || workspace_bytes < need)) return FAIRY2I_ERR_WORKSPACE;
+  if (need > 0 && !aligned(workspace, 16)) return FAIRY2I_ERR_ALIGNMENT;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int per = chain_max_calls();
+  for (int c0 = 0; c0 < ncalls; c0 += per) {
+    const int nc = ncalls - c0 < per ? ncalls - c0 : per;
+    unsigned int* done = nullptr;
+    if (nc > 1) {
+      done = static_cast<unsigned int*>(workspace);
+      if (cudaMemsetAsync(done, 0, (size_t)nc * sizeof(unsigned int), s) != cudaSuccess)
+        return FAIRY2I_ERR_CUDA;
+    }
+    const fairy2i_status st = launch_wl_chain(calls + c0, nc, T, cluster_size, done, s);
+    if (st != FAIRY2I_OK) return st;
+  }
+  return FAIRY2I_OK;
 }
 
 fairy2i_status fairy2i_codes_adjoint(const uint32_t* codes, int64_t n, int64_t m, int T,

@@ -90,7 +90,9 @@ def test_wl_matmul_validation(lib):
         return lib.fairy2i_wl_matmul_path(x, xdt, B, inf, ldx, codes, scales, outf, T, y, ldy,
                                           path, None)
     assert call(B=0) == 0                      # empty batch: nothing to do
-    assert call(B=-1) == 1 and call(T=0) == 1 and call(path=5) == 1 and call(x=None) == 1
+    assert call(B=-1) == 1 and call(T=0) == 1 and call(path=6) == 1 and call(x=None) == 1
+    assert call(path=2) == 1                   # retired
+    assert call(path=5, B=2) == 1 and call(path=5, T=5) == 1   # the chained kernel: one token, T <= 4
     assert call(xdt=7) == 4
     assert call(ldx=15) == 2 and call(ldy=15) == 2
     assert call(x=ODD) == 3 and call(codes=ODD) == 3
@@ -120,9 +122,9 @@ def test_wl_matmul_group_validation(lib):
     assert call(ldx=15) == 2 and call(ldy=15) == 2
     assert call(codes=arr(GOOD, ODD, GOOD, GOOD)) == 3        # a misaligned member
     assert call(ys=arr(GOOD, GOOD, None, GOOD)) == 1          # a null member
-    # the group call with an explicit kernel: only paths 0, 1 and 4 exist for a group
+    # the group call with an explicit kernel: only paths 0, 1, 4 and 5 exist for a group
     cp = arr(*([GOOD] * 4))
-    for path in (2, 3, 5, -1):
+    for path in (2, 3, 6, -1):
         assert lib.fairy2i_wl_matmul_group_path(GOOD, 1, 1, 16, 16, 3, cp, cp, 16, 2, cp, 16,
                                                 path, None) == 1
     assert lib.fairy2i_wl_matmul_group_path(GOOD, 1, 0, 16, 16, 3, cp, cp, 16, 2, cp, 16, 4,
@@ -135,3 +137,38 @@ def test_codes_adjoint_validation(lib):
     assert lib.fairy2i_codes_adjoint(GOOD, 4, 4, 9, P((1 << 24)), None) == 1
     assert lib.fairy2i_codes_adjoint(ODD, 4, 4, 2, P((1 << 24)), None) == 3
     assert lib.fairy2i_codes_adjoint(GOOD, 4, 4, 2, GOOD, None) == 1     # overlapping buffers
+
+
+def test_wl_matmul_chain_validation(lib):
+    """The chained decode refuses bad calls before anything is enqueued."""
+    from paper_2512_02901_gb300.binding import ChainCall
+    assert lib.fairy2i_wl_matmul_chain_max_calls() >= 128
+    assert lib.fairy2i_wl_matmul_chain_workspace_bytes(1) == 0
+    assert lib.fairy2i_wl_matmul_chain_workspace_bytes(128) >= 128 * 4
+
+    def good():
+        k = ChainCall()
+        k.x, k.xdt, k.count, k.in_features, k.out_features = GOOD, 1, 1, 4096, 4096
+        k.codes[0] = k.scales[0] = k.y[0] = GOOD
+        return k
+
+    def call(mod=None, n=1, T=2, cluster=0, ws=GOOD, wsb=1 << 20):
+        arr = (ChainCall * n)(*[good() for _ in range(n)])
+        if mod:
+            mod(arr[n - 1])
+        return lib.fairy2i_wl_matmul_chain(ctypes.cast(arr, ctypes.c_void_p), n, T, cluster, ws,
+                                           wsb, None)
+
+    assert call(T=0) == 1 and call(T=5) == 1 and call(cluster=3) == 1
+    assert lib.fairy2i_wl_matmul_chain(None, 1, 2, 0, None, 0, None) == 1
+    assert call(lambda k: setattr(k, "count", 0)) == 1
+    assert call(lambda k: setattr(k, "count", 5)) == 1
+    assert call(lambda k: setattr(k, "in_features", 24577)) == 1     # longer rows than the kernel takes
+    assert call(lambda k: setattr(k, "x", None)) == 1
+    assert call(lambda k: setattr(k, "xdt", 7)) == 4
+    assert call(lambda k: setattr(k, "x", ODD)) == 3
+    assert call(lambda k: k.codes.__setitem__(0, ODD)) == 3
+    assert call(lambda k: k.y.__setitem__(0, None)) == 1
+    assert call(n=3, ws=None, wsb=0) == 5                        # counters need a workspace
+    assert call(n=3, wsb=8) == 5
+    assert call(n=3, ws=ODD) == 3
