@@ -296,6 +296,71 @@ fairy2i_status fairy2i_wl_matmul_chain(const fairy2i_chain_call* calls, int ncal
                                        void* stream);
 
 /* ------------------------------------------------------------------------------------------
+ * The rest of a widely-linear decoder layer for one token (Sec. 3.1, self-attention in
+ * widely-linear form). Vectors use the real layout of the matmul calls: a complex vector of n
+ * channels is 2 n floats [Re | Im].
+ *
+ * Attention with Hermitian scores (Eq. hermitian-score) of one query over L cached positions:
+ *   head h is the complex channels [h dc, (h+1) dc), dc = n / heads, d_k = 2 dc;
+ *   S[h, l] = Re(q_h^H k_{l,h}) / sqrt(d_k) (the real dot product of the stacked head vectors),
+ *   p = softmax over l per head, o_h = sum_l p[h, l] v_{l,h} (real and imaginary parts of v
+ *   weighted alike).
+ *   q        float32 [2 n]; k_cache, v_cache float32 [L][ldkv] (2 n used per position: a key or
+ *            value as fairy2i_wl_matmul writes it, so a call can write the new position's key
+ *            and value straight into the caches); out float32 [2 n] (may not overlap the inputs).
+ *   workspace >= fairy2i_hermitian_attention_workspace_bytes(n, heads, L) bytes, 4-byte aligned
+ *            (per-split partial softmax sums; contents on entry do not matter).
+ *   Requirements: L >= 1, heads >= 1, n % heads == 0, dc <= 128, ldkv >= 2 n, pointers 4-byte
+ *   aligned. Scores and value sums are accumulated in two-float (compensated) arithmetic.
+ *   A real model's head layout (2 dc consecutive real channels per head) maps onto this one by
+ *   permuting the output channels of R_Q, R_K, R_V (and the input channels of R_O) before
+ *   conversion so that each head's real channels are the real and imaginary parts of dc complex
+ *   channels.
+ * ------------------------------------------------------------------------------------------ */
+size_t fairy2i_hermitian_attention_workspace_bytes(int64_t n, int heads, int64_t L);
+fairy2i_status fairy2i_hermitian_attention(const float* q, const float* k_cache,
+                                           const float* v_cache, int64_t L, int64_t ldkv,
+                                           int64_t n, int heads, float* out, void* workspace,
+                                           size_t workspace_bytes, void* stream);
+
+/* RMS normalisation of B tokens of d real values (the decoder's norm layers stay real): with
+ * v = h + delta (delta may be NULL), out = v / sqrt(mean(v^2) + eps) * w, and h_out = v when
+ * h_out is not NULL (the residual stream after an add). float32 throughout; out and h_out may
+ * alias h. Requirements: B >= 1, d >= 1, eps >= 0, pointers 4-byte aligned. */
+fairy2i_status fairy2i_rmsnorm(const float* h, const float* delta, const float* w, int64_t B,
+                               int64_t d, float eps, float* h_out, float* out, void* stream);
+
+/* The gated activation of the decoder's MLP, out = silu(g) * u elementwise over `count` float32
+ * values (out may alias g or u). */
+fairy2i_status fairy2i_silu_mul(const float* g, const float* u, int64_t count, float* out,
+                                void* stream);
+
+/* ------------------------------------------------------------------------------------------
+ * Host (CPU) matmul by look-up tables (Sec. 3.4, LUT-based optimization for CPU), for the host
+ * cores of the machine (no GPU involved; every pointer here is HOST memory).
+ * fairy2i_lut_quantize_x: int8 activations of one token, per-token symmetric absmax:
+ *   delta = float(max |x~_i| / 127) (float32 division), xq_i = round-half-even(x~_i / delta)
+ *   clamped to [-127, 127] (all zero when x~ = 0). x float32 [in_features], xq int8
+ *   [in_features]; *scale = delta. FAIRY2I_ERR_INVALID_ARG for a non-finite x.
+ * fairy2i_lut_matmul: y = delta sum_t (U^(t) z + W^(t) conj(z)), z the complex int8 token
+ *   (Re = xq[0:m], Im = xq[m:in_features], zero-padded), codes and scales as fairy2i_quantize
+ *   writes them (packed layout, HOST copies), y float32 [out_features] in the real layout.
+ *   Four codes of a packed word form one 8-bit index; per group of four inputs a table of 256
+ *   entries holds the exact integer partial sums over the real-axis codes and over the
+ *   imaginary-axis codes, one table serving U (z) and W (conj(z)). Sums are exact integers,
+ *   then scaled in float64: y equals the float64 widely-linear matmul of delta xq to rounding.
+ *   workspace >= fairy2i_lut_workspace_bytes(in_features) bytes of host memory (8-byte
+ *   aligned); nthreads host threads (1 .. 1024) split the tables and the rows.
+ * ------------------------------------------------------------------------------------------ */
+fairy2i_status fairy2i_lut_quantize_x(const float* x, int64_t in_features, int8_t* xq,
+                                      float* scale);
+size_t fairy2i_lut_workspace_bytes(int64_t in_features);
+fairy2i_status fairy2i_lut_matmul(const int8_t* xq, float x_scale, int64_t in_features,
+                                  const uint32_t* codes, const float* scales,
+                                  int64_t out_features, int T, float* y, void* workspace,
+                                  size_t workspace_bytes, int nthreads);
+
+/* ------------------------------------------------------------------------------------------
  * Synchronizes `stream`, then returns and clears the device-side status of the current
  * device: FAIRY2I_ERR_NONFINITE, FAIRY2I_ERR_TIMEOUT, FAIRY2I_ERR_CUDA (an asynchronous CUDA
  * error) or FAIRY2I_OK.

@@ -37,7 +37,8 @@ __all__ = [
     "complex_dims", "convert", "realify_lin", "realify_conj", "project", "fixed_tree_sum",
     "axis_scales", "dequant", "residual_quantize", "quantize", "words_per_row", "row_tiles",
     "pack_codes", "unpack_codes", "split_input", "wl_matmul", "wl_matmul_rows", "dense_realified",
-    "tolerance_bound", "adjoint_codes",
+    "tolerance_bound", "adjoint_codes", "hermitian_scores", "hermitian_attention", "rmsnorm",
+    "silu_mul", "decoder_layer", "quantize_activations_int8",
 ]
 
 F32 = np.float32
@@ -357,3 +358,94 @@ def tolerance_bound(x, scales):
     sc = np.asarray(scales, dtype=np.float64)
     s_sum = float(np.sum(np.max(sc, axis=2)))
     return np.abs(x).sum(axis=1) * s_sum
+
+
+# --------------------------------------------------------------------------------------------
+# Sec. 3.1 (self-attention in widely-linear form) -- Hermitian attention and a decoder layer
+# --------------------------------------------------------------------------------------------
+def hermitian_scores(q, K, heads: int):
+    """Eq. hermitian-score for one query token: S[h, l] = Re(q_h^H k_{l,h}) / sqrt(d_k).
+
+    q complex [n], K complex [L][n]; head h is the complex channels [h dc, (h+1) dc) with
+    dc = n / heads, and d_k = 2 dc is the head's real dimension (its stacked vector
+    [Re q_h ; Im q_h]). Returns float64 [heads][L]."""
+    q = np.asarray(q, dtype=np.complex128)
+    K = np.asarray(K, dtype=np.complex128)
+    n = q.shape[0]
+    dc = n // heads
+    qh = q.reshape(heads, dc)
+    Kh = K.reshape(K.shape[0], heads, dc)
+    return np.real(np.einsum("hc,lhc->hl", np.conj(qh), Kh)) / np.sqrt(2.0 * dc)
+
+
+def hermitian_attention(q, K, V, heads: int):
+    """Attention of one query over L keys/values with Hermitian scores (Eq. hermitian-score):
+    softmax over l of S[h, l] per head, then o_h = sum_l p[h, l] v_{l,h}; the weights are real,
+    so the real and imaginary parts of v are aggregated separately. Returns complex [n]."""
+    S = hermitian_scores(q, K, heads)
+    P = np.exp(S - S.max(axis=1, keepdims=True))
+    P /= P.sum(axis=1, keepdims=True)
+    V = np.asarray(V, dtype=np.complex128)
+    L, n = V.shape
+    dc = n // heads
+    return np.einsum("hl,lhc->hc", P, V.reshape(L, heads, dc)).reshape(n)
+
+
+def rmsnorm(h, w, eps: float):
+    """Root-mean-square normalisation of a real vector (the decoder's norm layers stay real:
+    the widely-linear rewrite concerns the linear maps only). h, w [d] -> h w / sqrt(mean h^2 + eps)."""
+    h = np.asarray(h, dtype=np.float64)
+    return h / np.sqrt(np.mean(h * h) + eps) * np.asarray(w, dtype=np.float64)
+
+
+def silu_mul(g, u):
+    """silu(g) * u, the gated activation of the decoder's MLP (real, elementwise)."""
+    g = np.asarray(g, dtype=np.float64)
+    return g / (1.0 + np.exp(-g)) * np.asarray(u, dtype=np.float64)
+
+
+def decoder_layer(h, layer, K_cache, V_cache, heads: int, eps: float = 1e-5):
+    """One decoder layer for one token (real layout h [d], d = 2 n), every linear the quantized
+    widely-linear map (Eq. widely-linear + Eq. res-sum, dequantized by Eq. ifairy-dequant) and
+    attention with Hermitian scores (Eq. hermitian-score):
+        x = rmsnorm(h) w_attn; q, k, v = Q x, K x, V x (complex); keys/values = cache + (k, v)
+        h1 = h + O [Re a ; Im a],  a = attention(q, keys, values)
+        x2 = rmsnorm(h1) w_mlp;  h2 = h1 + Down (silu(Gate x2) * Up x2)
+    `layer`: dict of (codes, scales) for q, k, v, o, gate, up, down (out/in features implied by
+    the codes' shapes) plus w_attn, w_mlp. K_cache, V_cache complex [L][n] (may be empty).
+    Returns h2 (float64 [d]) and the new key and value (complex [n])."""
+    def lin(name, x, out_features):
+        codes, scales = layer[name]
+        return wl_matmul(np.asarray(x, np.float64)[None, :], codes, scales, out_features)[0]
+    h = np.asarray(h, dtype=np.float64)
+    d = h.shape[0]
+    n = d // 2
+    x = rmsnorm(h, layer["w_attn"], eps)
+    q, k, v = (lin(nm, x, d) for nm in ("q", "k", "v"))
+    cq, ck, cv = (t[:n] + 1j * t[n:] for t in (q, k, v))
+    Kc = np.concatenate([np.asarray(K_cache, np.complex128).reshape(-1, n), ck[None, :]])
+    Vc = np.concatenate([np.asarray(V_cache, np.complex128).reshape(-1, n), cv[None, :]])
+    a = hermitian_attention(cq, Kc, Vc, heads)
+    h1 = h + lin("o", np.concatenate([a.real, a.imag]), d)
+    x2 = rmsnorm(h1, layer["w_mlp"], eps)
+    dff = 2 * np.shape(layer["gate"][0])[2]
+    m = silu_mul(lin("gate", x2, dff), lin("up", x2, dff))
+    h2 = h1 + lin("down", m, d)
+    return h2, ck, cv
+
+
+# --------------------------------------------------------------------------------------------
+# Sec. 3.4 (LUT-based optimization for CPU) -- int8 activations
+# --------------------------------------------------------------------------------------------
+def quantize_activations_int8(x):
+    """int8 activations for the table-lookup matmul (the paper names INT8 activations without
+    fixing the quantizer; read here as per-token symmetric absmax): delta = max|x~| / 127 as one
+    float32 division, xq = round-half-even(x~ / delta) in float32, clamped to [-127, 127]; a zero
+    token gives delta = 0 and xq = 0. x [in_features] -> (xq int8, delta float32)."""
+    x = np.asarray(x, dtype=F32).ravel()
+    mx = F32(np.max(np.abs(x))) if x.size else F32(0)
+    delta = F32(mx / F32(127))
+    if delta == 0:
+        return np.zeros(x.shape, np.int8), delta
+    q = np.rint(x / delta).astype(F32)
+    return np.clip(q, -127, 127).astype(np.int8), delta

@@ -52,6 +52,15 @@ class ChainCall(ctypes.Structure):
 
 
 SIGNATURES.update({
+    "fairy2i_hermitian_attention_workspace_bytes": ([_i64, _int, _i64], _sz),
+    "fairy2i_hermitian_attention": ([_vp, _vp, _vp, _i64, _i64, _i64, _int, _vp, _vp, _sz, _vp],
+                                    _int),
+    "fairy2i_rmsnorm": ([_vp, _vp, _vp, _i64, _i64, _c.c_float, _vp, _vp, _vp], _int),
+    "fairy2i_silu_mul": ([_vp, _vp, _i64, _vp, _vp], _int),
+    "fairy2i_lut_quantize_x": ([_vp, _i64, _vp, _vp], _int),
+    "fairy2i_lut_workspace_bytes": ([_i64], _sz),
+    "fairy2i_lut_matmul": ([_vp, _c.c_float, _i64, _vp, _vp, _i64, _int, _vp, _vp, _sz, _int],
+                           _int),
     "fairy2i_wl_matmul_chain_max_calls": ([], _int),
     "fairy2i_wl_matmul_chain_workspace_bytes": ([_int], _sz),
     "fairy2i_wl_matmul_chain": ([_vp, _int, _int, _int, _vp, _sz, _vp], _int),
@@ -281,6 +290,90 @@ def wl_matmul_chain(calls, T: int, cluster_size: int = 0, workspace=None, stream
     return arr
 
 
+def hermitian_attention(q: torch.Tensor, k_cache: torch.Tensor, v_cache: torch.Tensor, L: int,
+                        heads: int, out=None, workspace=None, stream=None) -> torch.Tensor:
+    """Attention of one query over the first L cached positions with Hermitian scores
+    (fairy2i_hermitian_attention). q float32 [2 n] ([Re | Im]); caches float32 [Lmax][2 n]
+    (rows as wl_matmul writes them); returns float32 [2 n]."""
+    assert q.is_cuda and q.dtype == torch.float32 and q.is_contiguous()
+    for c in (k_cache, v_cache):
+        assert c.is_cuda and c.dtype == torch.float32 and c.dim() == 2 and c.stride(1) == 1
+        assert c.shape[0] >= L and c.shape[1] >= q.numel()
+    n = q.numel() // 2
+    if out is None:
+        out = torch.empty(2 * n, dtype=torch.float32, device=q.device)
+    nbytes = int(load().fairy2i_hermitian_attention_workspace_bytes(n, heads, L))
+    if workspace is None or workspace.numel() < nbytes:
+        workspace = torch.empty(max(nbytes, 4), dtype=torch.uint8, device=q.device)
+    _check("fairy2i_hermitian_attention",
+           load().fairy2i_hermitian_attention(_ptr(q), _ptr(k_cache), _ptr(v_cache), L,
+                                              k_cache.stride(0), n, heads, _ptr(out),
+                                              _ptr(workspace), workspace.numel(), _stream(stream)))
+    return out
+
+
+def rmsnorm(h: torch.Tensor, w: torch.Tensor, eps: float, delta=None, h_out=None, out=None,
+            stream=None) -> torch.Tensor:
+    """out = (h + delta) / sqrt(mean((h + delta)^2) + eps) * w per token (fairy2i_rmsnorm);
+    h_out, if given, receives h + delta. h [B][d] float32 (CUDA)."""
+    assert h.is_cuda and h.dtype == torch.float32 and h.is_contiguous()
+    h2 = h.view(-1, h.shape[-1])
+    B, d = h2.shape
+    assert w.numel() == d and w.dtype == torch.float32 and w.is_contiguous()
+    if delta is not None:
+        assert delta.shape == h.shape and delta.dtype == torch.float32 and delta.is_contiguous()
+    if out is None:
+        out = torch.empty_like(h)
+    _check("fairy2i_rmsnorm",
+           load().fairy2i_rmsnorm(_ptr(h), _ptr(delta) if delta is not None else None, _ptr(w), B,
+                                  d, eps, _ptr(h_out) if h_out is not None else None, _ptr(out),
+                                  _stream(stream)))
+    return out
+
+
+def silu_mul(g: torch.Tensor, u: torch.Tensor, out=None, stream=None) -> torch.Tensor:
+    """silu(g) * u elementwise (fairy2i_silu_mul), float32 CUDA tensors of the same size."""
+    assert g.is_cuda and g.dtype == torch.float32 and g.is_contiguous() and u.shape == g.shape
+    if out is None:
+        out = torch.empty_like(g)
+    _check("fairy2i_silu_mul", load().fairy2i_silu_mul(_ptr(g), _ptr(u), g.numel(), _ptr(out),
+                                                       _stream(stream)))
+    return out
+
+
+def lut_quantize_x(x: torch.Tensor):
+    """int8 activations of one token on the host (fairy2i_lut_quantize_x): returns (xq, delta)."""
+    x = x.detach().to("cpu", torch.float32).contiguous().view(-1)
+    xq = torch.empty(x.numel(), dtype=torch.int8)
+    sc = ctypes.c_float()
+    _check("fairy2i_lut_quantize_x",
+           load().fairy2i_lut_quantize_x(_ptr(x), x.numel(), _ptr(xq), ctypes.byref(sc)))
+    return xq, float(sc.value)
+
+
+def lut_matmul(xq: torch.Tensor, delta: float, codes: torch.Tensor, scales: torch.Tensor,
+               out_features: int, T: int | None = None, nthreads: int | None = None,
+               workspace=None) -> torch.Tensor:
+    """The host look-up-table matmul (fairy2i_lut_matmul) of one int8 token: host tensors."""
+    assert xq.dtype == torch.int8 and not xq.is_cuda and xq.is_contiguous()
+    codes = codes.detach().to("cpu").contiguous()
+    scales = scales.detach().to("cpu", torch.float32).contiguous()
+    in_features = xq.numel()
+    if T is None:
+        T = scales.shape[0]
+    check_layer(codes, scales, out_features, in_features, T)
+    nbytes = int(load().fairy2i_lut_workspace_bytes(in_features))
+    if workspace is None or workspace.numel() < nbytes:
+        workspace = torch.empty(nbytes, dtype=torch.uint8)
+    y = torch.empty(out_features, dtype=torch.float32)
+    nthreads = nthreads or (os.cpu_count() or 1)
+    _check("fairy2i_lut_matmul",
+           load().fairy2i_lut_matmul(_ptr(xq), delta, in_features, _ptr(codes), _ptr(scales),
+                                     out_features, T, _ptr(y), _ptr(workspace), workspace.numel(),
+                                     nthreads))
+    return y
+
+
 def codes_adjoint(codes: torch.Tensor, n: int, m: int, T: int, stream=None) -> torch.Tensor:
     """Codes of the adjoint layer (input gradient, R^T): the layout fairy2i_quantize writes for
     an m x n layer. wl_matmul(y_grad, codes_adjoint(...), scales, in_features) = x~_grad."""
@@ -329,3 +422,61 @@ class Fairy2iLinear:
         layer.codes, layer.scales, layer.out_features, layer.in_features, layer.T = \
             artifact.load(path, device)
         return layer
+
+
+class WLDecoderLayer:
+    """A decoder layer whose seven linears are quantized widely-linear maps and whose attention
+    uses Hermitian scores (Sec. 3.1), for one token at a time with a key/value cache. Every step
+    is a library call on the device: RMS norm (with the residual add of the previous sub-layer
+    fused in), the grouped q/k/v matmul writing the new key and value straight into the caches,
+    attention, o, gate/up, silu * up, down. Activations are float32 (the chained decode kernel).
+
+    step(h, delta) takes the residual stream as h + delta and returns (h1, d) with the layer's
+    output h1 + d, so the next layer (or a final norm) fuses that add too."""
+
+    NAMES = ("q", "k", "v", "o", "gate", "up", "down")
+
+    def __init__(self, weights: dict, w_attn: torch.Tensor, w_mlp: torch.Tensor, heads: int,
+                 max_len: int, T: int = 2, eps: float = 1e-5):
+        self.d = weights["q"].shape[1]
+        self.dff = weights["gate"].shape[0]
+        self.heads, self.T, self.eps, self.max_len = heads, T, eps, max_len
+        dev = weights["q"].device
+        self.codes, self.scales = {}, {}
+        for nm in self.NAMES:
+            U, W = convert(weights[nm])
+            self.codes[nm], self.scales[nm] = quantize(U, W, T)
+        self.w_attn, self.w_mlp = w_attn.contiguous(), w_mlp.contiguous()
+        self.k_cache = torch.zeros((max_len, self.d), dtype=torch.float32, device=dev)
+        self.v_cache = torch.zeros((max_len, self.d), dtype=torch.float32, device=dev)
+        self.pos = 0
+        f = lambda *s: torch.empty(s, dtype=torch.float32, device=dev)
+        self.x, self.q, self.a, self.o = f(1, self.d), f(1, self.d), f(1, self.d), f(1, self.d)
+        self.h1, self.x2 = f(1, self.d), f(1, self.d)
+        self.g, self.u, self.m = f(1, self.dff), f(1, self.dff), f(1, self.dff)
+        self.dn = f(1, self.d)
+        self.ws = torch.empty(max(int(load().fairy2i_hermitian_attention_workspace_bytes(
+            self.d // 2, heads, max_len)), 4), dtype=torch.uint8, device=dev)
+
+    def step(self, h: torch.Tensor, delta=None, stream=None):
+        assert self.pos < self.max_len
+        p = self.pos
+        rmsnorm(h, self.w_attn, self.eps, delta=delta, h_out=h if delta is not None else None,
+                out=self.x, stream=stream)
+        wl_matmul_group(self.x, [self.codes[n] for n in ("q", "k", "v")],
+                        [self.scales[n] for n in ("q", "k", "v")], self.d,
+                        ys=[self.q, self.k_cache[p:p + 1], self.v_cache[p:p + 1]],
+                        path=PATH_CHAIN, stream=stream, T=self.T)
+        hermitian_attention(self.q.view(-1), self.k_cache, self.v_cache, p + 1, self.heads,
+                            out=self.a.view(-1), workspace=self.ws, stream=stream)
+        wl_matmul(self.a, self.codes["o"], self.scales["o"], self.d, y=self.o, path=PATH_CHAIN,
+                  stream=stream, T=self.T)
+        rmsnorm(h, self.w_mlp, self.eps, delta=self.o, h_out=self.h1, out=self.x2, stream=stream)
+        wl_matmul_group(self.x2, [self.codes["gate"], self.codes["up"]],
+                        [self.scales["gate"], self.scales["up"]], self.dff, ys=[self.g, self.u],
+                        path=PATH_CHAIN, stream=stream, T=self.T)
+        silu_mul(self.g, self.u, out=self.m, stream=stream)
+        wl_matmul(self.m, self.codes["down"], self.scales["down"], self.d, y=self.dn,
+                  path=PATH_CHAIN, stream=stream, T=self.T)
+        self.pos += 1
+        return self.h1, self.dn

@@ -36,6 +36,14 @@ fairy2i_status launch_selftest_wait(uint32_t limit_us, cudaStream_t stream);
 fairy2i_status launch_wl_chain(const fairy2i_chain_call* calls, int ncalls, int T,
                                int cluster_size, unsigned int* done, cudaStream_t stream);
 int chain_max_calls();
+size_t attention_workspace_bytes(int64_t n, int heads, int64_t L);
+fairy2i_status launch_attention(const float* q, const float* kc, const float* vc, int64_t L,
+                                int64_t ldkv, int64_t n, int heads, float* out, void* ws,
+                                size_t ws_bytes, cudaStream_t stream);
+fairy2i_status launch_rmsnorm(const float* h, const float* delta, const float* w, int64_t B,
+                              int64_t d, float eps, float* h_out, float* out, cudaStream_t stream);
+fairy2i_status launch_silu_mul(const float* g, const float* u, int64_t count, float* out,
+                               cudaStream_t stream);
 fairy2i_status launch_codes_adjoint(const uint32_t* codes, int64_t n, int64_t m, int T,
                                     uint32_t* codes_adj, cudaStream_t stream);
 fairy2i_status launch_wl_decode_group(const void* x, fairy2i_dtype xdt, int64_t B,
@@ -323,6 +331,44 @@ fairy2i_status fairy2i_wl_matmul_chain(const fairy2i_chain_call* calls, int ncal
     if (st != FAIRY2I_OK) return st;
   }
   return FAIRY2I_OK;
+}
+
+size_t fairy2i_hermitian_attention_workspace_bytes(int64_t n, int heads, int64_t L) {
+  return attention_workspace_bytes(n, heads, L);
+}
+
+fairy2i_status fairy2i_hermitian_attention(const float* q, const float* k_cache,
+                                           const float* v_cache, int64_t L, int64_t ldkv,
+                                           int64_t n, int heads, float* out, void* workspace,
+                                           size_t workspace_bytes, void* stream) {
+  if (!q || !k_cache || !v_cache || !out || L < 1 || n < 1 || heads < 1 || n % heads != 0 ||
+      n / heads > 128)
+    return FAIRY2I_ERR_INVALID_ARG;
+  if (ldkv < 2 * n) return FAIRY2I_ERR_SHAPE;
+  if (!aligned(q, 4) || !aligned(k_cache, 4) || !aligned(v_cache, 4) || !aligned(out, 4))
+    return FAIRY2I_ERR_ALIGNMENT;
+  if (!workspace || workspace_bytes < attention_workspace_bytes(n, heads, L))
+    return FAIRY2I_ERR_WORKSPACE;
+  if (!aligned(workspace, 4)) return FAIRY2I_ERR_ALIGNMENT;
+  return launch_attention(q, k_cache, v_cache, L, ldkv, n, heads, out, workspace, workspace_bytes,
+                          static_cast<cudaStream_t>(stream));
+}
+
+fairy2i_status fairy2i_rmsnorm(const float* h, const float* delta, const float* w, int64_t B,
+                               int64_t d, float eps, float* h_out, float* out, void* stream) {
+  if (!h || !w || !out || B < 1 || d < 1 || !(eps >= 0.f) || B > (int64_t(1) << 31))
+    return FAIRY2I_ERR_INVALID_ARG;
+  if (!aligned(h, 4) || !aligned(w, 4) || !aligned(out, 4) || (delta && !aligned(delta, 4)) ||
+      (h_out && !aligned(h_out, 4)))
+    return FAIRY2I_ERR_ALIGNMENT;
+  return launch_rmsnorm(h, delta, w, B, d, eps, h_out, out, static_cast<cudaStream_t>(stream));
+}
+
+fairy2i_status fairy2i_silu_mul(const float* g, const float* u, int64_t count, float* out,
+                                void* stream) {
+  if (!g || !u || !out || count < 1) return FAIRY2I_ERR_INVALID_ARG;
+  if (!aligned(g, 4) || !aligned(u, 4) || !aligned(out, 4)) return FAIRY2I_ERR_ALIGNMENT;
+  return launch_silu_mul(g, u, count, out, static_cast<cudaStream_t>(stream));
 }
 
 fairy2i_status fairy2i_codes_adjoint(const uint32_t* codes, int64_t n, int64_t m, int T,
