@@ -361,6 +361,47 @@ fairy2i_status fairy2i_lut_matmul(const int8_t* xq, float x_scale, int64_t in_fe
                                   size_t workspace_bytes, int nthreads);
 
 /* ------------------------------------------------------------------------------------------
+ * Gradients for quantization-aware training (Sec. 3.2 QAT paragraph, Sec. 3.3 QAT).
+ *
+ * fairy2i_ste_weight_grad: the gradient of a loss with respect to the dequantized pair (U^, W^)
+ *   of a layer, which the straight-through estimator passes to the full-precision masters:
+ *   dU = sum_b g_b conj(x_b)^T, dW = sum_b g_b x_b^T (complex), from y = U^ x + W^ conj(x).
+ *   x   bf16 [B][ldx] real layout (in_features used), the layer input;
+ *   g   bf16 [B][ldg] real layout (out_features used), dL/dy~;
+ *   dU, dW complex64 [n][ldc] (n = ceil(out/2), m = ceil(in/2), ldc >= m), written, or added
+ *   to when accumulate != 0. One real GEMM G = g~^T x~ on the tensor cores (bf16 x bf16 -> f32)
+ *   gives both: dU = (G11 + G22) + i (G21 - G12), dW = (G11 - G22) + i (G12 + G21).
+ *   workspace >= fairy2i_ste_weight_grad_workspace_bytes(B, in_features, out_features) bytes,
+ *   256-byte aligned (token-contiguous copies of x and g). Requirements: B, in, out >= 1,
+ *   x, g 2-byte aligned, dU, dW 8-byte aligned.
+ *
+ * fairy2i_scale_grad: the part of the master gradient that flows through the per-tensor scales
+ *   of Eq. ifairy-scale, codes held fixed. For M in {U, W} with dM = dL/dM^ (e.g. from
+ *   fairy2i_ste_weight_grad), backpropagating through r^(t+1) = r^(t) - (s_re b_re + i s_im b_im)
+ *   and s_re = mean |Re r^(t)| over the +-1 codes (s_im likewise) gives, from r^_T = 0,
+ *     s^_t = <dM - r^_(t+1), b^t> (real parts over the +-1 codes, imaginary over the +-i codes),
+ *     r^_t = r^_(t+1) + s^_re,t sign(Re r^(t)) / N_re [+-1 codes] + i s^_im,t sign(Im r^(t)) /
+ *            N_im [+-i codes];
+ *   gU, gW (complex64 [n][ldr]) receive r^_0, shat (float32 [T][2][2]) the total scale
+ *   gradients s^. The full master gradient is dM + r^_0. U, W, codes, scales as fairy2i_quantize
+ *   read and wrote them (r^(t) is replayed exactly as the quantizer computed it); sums are
+ *   float64 in a fixed order. workspace >= fairy2i_scale_grad_workspace_bytes() bytes, 8-byte
+ *   aligned. Requirements: n, m >= 1, 1 <= T <= 8, ldc, ldg, ldr >= m.
+ * ------------------------------------------------------------------------------------------ */
+size_t fairy2i_ste_weight_grad_workspace_bytes(int64_t B, int64_t in_features,
+                                               int64_t out_features);
+fairy2i_status fairy2i_ste_weight_grad(const void* x, int64_t ldx, const void* g, int64_t ldg,
+                                       int64_t B, int64_t in_features, int64_t out_features,
+                                       float* dU, float* dW, int64_t ldc, int accumulate,
+                                       void* workspace, size_t workspace_bytes, void* stream);
+size_t fairy2i_scale_grad_workspace_bytes(void);
+fairy2i_status fairy2i_scale_grad(const float* U, const float* W, int64_t n, int64_t m,
+                                  int64_t ldc, int T, const uint32_t* codes, const float* scales,
+                                  const float* dU, const float* dW, int64_t ldg, float* gU,
+                                  float* gW, int64_t ldr, float* shat, void* workspace,
+                                  size_t workspace_bytes, void* stream);
+
+/* ------------------------------------------------------------------------------------------
  * Synchronizes `stream`, then returns and clears the device-side status of the current
  * device: FAIRY2I_ERR_NONFINITE, FAIRY2I_ERR_TIMEOUT, FAIRY2I_ERR_CUDA (an asynchronous CUDA
  * error) or FAIRY2I_OK.

@@ -38,7 +38,8 @@ __all__ = [
     "axis_scales", "dequant", "residual_quantize", "quantize", "words_per_row", "row_tiles",
     "pack_codes", "unpack_codes", "split_input", "wl_matmul", "wl_matmul_rows", "dense_realified",
     "tolerance_bound", "adjoint_codes", "hermitian_scores", "hermitian_attention", "rmsnorm",
-    "silu_mul", "decoder_layer", "quantize_activations_int8",
+    "silu_mul", "decoder_layer", "quantize_activations_int8", "ste_weight_grad",
+    "scale_path_grad",
 ]
 
 F32 = np.float32
@@ -449,3 +450,70 @@ def quantize_activations_int8(x):
         return np.zeros(x.shape, np.int8), delta
     q = np.rint(x / delta).astype(F32)
     return np.clip(q, -127, 127).astype(np.int8), delta
+
+
+# --------------------------------------------------------------------------------------------
+# Sec. 3.2 / 3.3 (QAT) -- gradients of the quantized layer
+# --------------------------------------------------------------------------------------------
+def ste_weight_grad(x, g, n: int, m: int):
+    """Gradient of a loss L with respect to the dequantized pair (U^, W^) of a layer, given the
+    layer input x~ [B][in_features] and the output gradient g~ = dL/dy~ [B][out_features] (real
+    layouts). From y = U^ x + W^ conj(x) (Eq. widely-linear), with complex gradients written as
+    dL/dRe + i dL/dIm: dU = sum_b g_b conj(x_b)^T and dW = sum_b g_b x_b^T (complex [n][m]). Under
+    the straight-through estimator (Sec. 3.2 QAT) this is the gradient passed to the masters."""
+    z = split_input(x, m)
+    gc = split_input(g, n)
+    return gc.T @ np.conj(z), gc.T @ z
+
+
+def scale_path_grad(M, codes_M, scales_M, dM, mode: str = "math"):
+    """The part of the master gradient that flows through the per-tensor scales (Eq.
+    ifairy-scale) of the T residual stages (Sec. 3.3), codes held fixed (straight-through), for
+    one matrix M (complex [n][m], float64) with its codes [T][n][m], scales [T][2] and the
+    gradient dM = dL/dM^ of the dequantized matrix (complex [n][m]). The loss is linear in the
+    scales: L = sum_t a_t s_re^t + c_t s_im^t with a_t = <Re dM, b_re^t>, c_t = <Im dM, b_im^t>.
+    Backward through r^(t+1) = r^(t) - (s_re^t b_re^t + i s_im^t b_im^t), r^(0) = M and
+    s_re^t = mean over the +-1 codes of |Re r^(t)| (s_im alike):
+        s^_t = (a_t, c_t) - <r^_(t+1), b^t> (real and imaginary parts separately),
+        r^_t = r^_(t+1) + s^_re,t sign(Re r^(t)) [c in {+-1}] / N_re + i (same for Im),
+    from r^_T = 0. Returns (r^_0 = dL/dM through the scales, complex [n][m], and the total scale
+    gradients s^ [T][2]). mode "contract" replays the residuals in float32 exactly as the
+    quantizer computes them (the library's replay); "math" in float64."""
+    codes_M = np.asarray(codes_M)
+    T = codes_M.shape[0]
+    if mode == "contract":
+        # the quantizer's own float32 residuals (one rounding per update)
+        re = np.array(np.real(M), dtype=F32)
+        im = np.array(np.imag(M), dtype=F32)
+        res = [re.astype(np.float64) + 1j * im.astype(np.float64)]
+        for t in range(T):
+            c = codes_M[t]
+            s_re, s_im = F32(scales_M[t][0]), F32(scales_M[t][1])
+            re = np.where(c == 0, re - s_re, np.where(c == 2, re + s_re, re)).astype(F32)
+            im = np.where(c == 1, im - s_im, np.where(c == 3, im + s_im, im)).astype(F32)
+            res.append(re.astype(np.float64) + 1j * im.astype(np.float64))
+        M = res[0]
+    else:
+        M = np.asarray(M, np.complex128)
+        res = [M.copy()]
+        for t in range(T):
+            w = dequant(codes_M[t], scales_M[t][0], scales_M[t][1])
+            res.append(res[-1] - w)
+    dM = np.asarray(dM, np.complex128)
+    rhat = np.zeros_like(M)
+    shat = np.zeros((T, 2))
+    for t in range(T - 1, -1, -1):
+        c = codes_M[t]
+        b_re = np.select([c == 0, c == 2], [1.0, -1.0], 0.0)
+        b_im = np.select([c == 1, c == 3], [1.0, -1.0], 0.0)
+        on_re = (c == 0) | (c == 2)
+        on_im = ~on_re
+        sre = float(np.sum(dM.real * b_re)) - float(np.sum(rhat.real * b_re))
+        sim = float(np.sum(dM.imag * b_im)) - float(np.sum(rhat.imag * b_im))
+        shat[t] = (sre, sim)
+        r = res[t]
+        n_re, n_im = int(on_re.sum()), int(on_im.sum())
+        add_re = np.where(on_re, np.sign(r.real) * sre / n_re, 0.0) if n_re else 0.0
+        add_im = np.where(on_im, np.sign(r.imag) * sim / n_im, 0.0) if n_im else 0.0
+        rhat = rhat + add_re + 1j * add_im
+    return rhat, shat

@@ -61,6 +61,12 @@ SIGNATURES.update({
     "fairy2i_lut_workspace_bytes": ([_i64], _sz),
     "fairy2i_lut_matmul": ([_vp, _c.c_float, _i64, _vp, _vp, _i64, _int, _vp, _vp, _sz, _int],
                            _int),
+    "fairy2i_ste_weight_grad_workspace_bytes": ([_i64, _i64, _i64], _sz),
+    "fairy2i_ste_weight_grad": ([_vp, _i64, _vp, _i64, _i64, _i64, _i64, _vp, _vp, _i64, _int,
+                                 _vp, _sz, _vp], _int),
+    "fairy2i_scale_grad_workspace_bytes": ([], _sz),
+    "fairy2i_scale_grad": ([_vp, _vp, _i64, _i64, _i64, _int, _vp, _vp, _vp, _vp, _i64, _vp, _vp,
+                            _i64, _vp, _vp, _sz, _vp], _int),
     "fairy2i_wl_matmul_chain_max_calls": ([], _int),
     "fairy2i_wl_matmul_chain_workspace_bytes": ([_int], _sz),
     "fairy2i_wl_matmul_chain": ([_vp, _int, _int, _int, _vp, _sz, _vp], _int),
@@ -372,6 +378,53 @@ def lut_matmul(xq: torch.Tensor, delta: float, codes: torch.Tensor, scales: torc
                                      out_features, T, _ptr(y), _ptr(workspace), workspace.numel(),
                                      nthreads))
     return y
+
+
+def ste_weight_grad(x: torch.Tensor, g: torch.Tensor, dU=None, dW=None, accumulate: bool = False,
+                    stream=None):
+    """dL/dU^, dL/dW^ (complex64 [n][m]) of a layer from its bf16 input x [B][in] and output
+    gradient g [B][out] (fairy2i_ste_weight_grad); added to dU, dW when accumulate."""
+    assert x.is_cuda and g.is_cuda and x.dtype == torch.bfloat16 and g.dtype == torch.bfloat16
+    assert x.dim() == 2 and g.dim() == 2 and x.shape[0] == g.shape[0]
+    assert x.stride(1) == 1 and g.stride(1) == 1
+    B, in_f = x.shape
+    out_f = g.shape[1]
+    n, m = complex_dims(out_f, in_f)
+    if dU is None:
+        dU = torch.zeros((n, m), dtype=torch.complex64, device=x.device)
+    if dW is None:
+        dW = torch.zeros((n, m), dtype=torch.complex64, device=x.device)
+    assert dU.shape == (n, m) and dW.shape == (n, m) and dU.is_contiguous() and dW.is_contiguous()
+    nb = int(load().fairy2i_ste_weight_grad_workspace_bytes(B, in_f, out_f))
+    ws = torch.empty(nb, dtype=torch.uint8, device=x.device)
+    _check("fairy2i_ste_weight_grad",
+           load().fairy2i_ste_weight_grad(_ptr(x), x.stride(0), _ptr(g), g.stride(0), B, in_f,
+                                          out_f, _ptr(torch.view_as_real(dU)),
+                                          _ptr(torch.view_as_real(dW)), m, int(accumulate),
+                                          _ptr(ws), nb, _stream(stream)))
+    return dU, dW
+
+
+def scale_grad(U: torch.Tensor, W: torch.Tensor, codes: torch.Tensor, scales: torch.Tensor,
+               dU: torch.Tensor, dW: torch.Tensor, T: int | None = None, stream=None):
+    """Master gradient through the scales (fairy2i_scale_grad): returns (gU, gW, shat) with
+    gU, gW complex64 [n][m] and shat float32 [T][2][2]."""
+    n, m = U.shape
+    if T is None:
+        T = scales.shape[0]
+    for t in (U, W, dU, dW):
+        assert t.is_cuda and t.dtype == torch.complex64 and t.shape == (n, m) and t.is_contiguous()
+    gU = torch.empty_like(U)
+    gW = torch.empty_like(W)
+    shat = torch.empty((T, 2, 2), dtype=torch.float32, device=U.device)
+    nb = int(load().fairy2i_scale_grad_workspace_bytes())
+    ws = torch.empty(nb, dtype=torch.uint8, device=U.device)
+    r = torch.view_as_real
+    _check("fairy2i_scale_grad",
+           load().fairy2i_scale_grad(_ptr(r(U)), _ptr(r(W)), n, m, m, T, _ptr(codes), _ptr(scales),
+                                     _ptr(r(dU)), _ptr(r(dW)), m, _ptr(r(gU)), _ptr(r(gW)), m,
+                                     _ptr(shat), _ptr(ws), nb, _stream(stream)))
+    return gU, gW, shat
 
 
 def codes_adjoint(codes: torch.Tensor, n: int, m: int, T: int, stream=None) -> torch.Tensor:

@@ -36,6 +36,15 @@ fairy2i_status launch_selftest_wait(uint32_t limit_us, cudaStream_t stream);
 fairy2i_status launch_wl_chain(const fairy2i_chain_call* calls, int ncalls, int T,
                                int cluster_size, unsigned int* done, cudaStream_t stream);
 int chain_max_calls();
+size_t ste_grad_workspace_bytes(int64_t B, int64_t in_features, int64_t out_features);
+fairy2i_status launch_ste_grad(const void* x, int64_t ldx, const void* g, int64_t ldg, int64_t B,
+                               int64_t in_features, int64_t out_features, float* dU, float* dW,
+                               int64_t ldc, int accumulate, void* ws, cudaStream_t stream);
+size_t scale_grad_workspace_bytes();
+fairy2i_status launch_scale_grad(const float* U, const float* W, int64_t n, int64_t m, int64_t ldc,
+                                 int T, const uint32_t* codes, const float* scales, const float* dU,
+                                 const float* dW, int64_t ldg, float* rU, float* rW, int64_t ldr,
+                                 float* shat, void* ws, cudaStream_t stream);
 size_t attention_workspace_bytes(int64_t n, int heads, int64_t L);
 fairy2i_status launch_attention(const float* q, const float* kc, const float* vc, int64_t L,
                                 int64_t ldkv, int64_t n, int heads, float* out, void* ws,
@@ -369,6 +378,52 @@ fairy2i_status fairy2i_silu_mul(const float* g, const float* u, int64_t count, f
   if (!g || !u || !out || count < 1) return FAIRY2I_ERR_INVALID_ARG;
   if (!aligned(g, 4) || !aligned(u, 4) || !aligned(out, 4)) return FAIRY2I_ERR_ALIGNMENT;
   return launch_silu_mul(g, u, count, out, static_cast<cudaStream_t>(stream));
+}
+
+size_t fairy2i_ste_weight_grad_workspace_bytes(int64_t B, int64_t in_features,
+                                               int64_t out_features) {
+  if (B < 1 || in_features < 1 || out_features < 1) return 0;
+  return ste_grad_workspace_bytes(B, in_features, out_features);
+}
+
+fairy2i_status fairy2i_ste_weight_grad(const void* x, int64_t ldx, const void* g, int64_t ldg,
+                                       int64_t B, int64_t in_features, int64_t out_features,
+                                       float* dU, float* dW, int64_t ldc, int accumulate,
+                                       void* workspace, size_t workspace_bytes, void* stream) {
+  if (!x || !g || !dU || !dW || B < 1 || in_features < 1 || out_features < 1 ||
+      B > (int64_t(1) << 26) || in_features > (int64_t(1) << 26) ||
+      out_features > (int64_t(1) << 26))
+    return FAIRY2I_ERR_INVALID_ARG;
+  const int64_t m = (in_features + 1) / 2;
+  if (ldx < in_features || ldg < out_features || ldc < m) return FAIRY2I_ERR_SHAPE;
+  if (!aligned(x, 2) || !aligned(g, 2) || !aligned(dU, 8) || !aligned(dW, 8))
+    return FAIRY2I_ERR_ALIGNMENT;
+  if (!workspace || workspace_bytes < ste_grad_workspace_bytes(B, in_features, out_features))
+    return FAIRY2I_ERR_WORKSPACE;
+  if (!aligned(workspace, 256)) return FAIRY2I_ERR_ALIGNMENT;
+  return launch_ste_grad(x, ldx, g, ldg, B, in_features, out_features, dU, dW, ldc, accumulate,
+                         workspace, static_cast<cudaStream_t>(stream));
+}
+
+size_t fairy2i_scale_grad_workspace_bytes(void) { return scale_grad_workspace_bytes(); }
+
+fairy2i_status fairy2i_scale_grad(const float* U, const float* W, int64_t n, int64_t m,
+                                  int64_t ldc, int T, const uint32_t* codes, const float* scales,
+                                  const float* dU, const float* dW, int64_t ldg, float* gU,
+                                  float* gW, int64_t ldr, float* shat, void* workspace,
+                                  size_t workspace_bytes, void* stream) {
+  if (!U || !W || !codes || !scales || !dU || !dW || !gU || !gW || !shat || n < 1 || m < 1 ||
+      T < 1 || T > FAIRY2I_MAX_STAGES)
+    return FAIRY2I_ERR_INVALID_ARG;
+  if (n > (int64_t(1) << 40) / m) return FAIRY2I_ERR_SHAPE;
+  if (ldc < m || ldg < m || ldr < m) return FAIRY2I_ERR_SHAPE;
+  if (!aligned(U, 8) || !aligned(W, 8) || !aligned(dU, 8) || !aligned(dW, 8) || !aligned(gU, 8) ||
+      !aligned(gW, 8) || !aligned(codes, 16) || !aligned(scales, 4) || !aligned(shat, 4))
+    return FAIRY2I_ERR_ALIGNMENT;
+  if (!workspace || workspace_bytes < scale_grad_workspace_bytes()) return FAIRY2I_ERR_WORKSPACE;
+  if (!aligned(workspace, 8)) return FAIRY2I_ERR_ALIGNMENT;
+  return launch_scale_grad(U, W, n, m, ldc, T, codes, scales, dU, dW, ldg, gU, gW, ldr, shat,
+                           workspace, static_cast<cudaStream_t>(stream));
 }
 
 fairy2i_status fairy2i_codes_adjoint(const uint32_t* codes, int64_t n, int64_t m, int T,
