@@ -36,10 +36,14 @@
 // c - 1's counter holds every cluster's arrival.
 //
 // Roles: warps 0-7 are two decoder sets of four (warp w reaches TMEM lanes 32 (w % 4) ..), set s
-// decoding units q = s, s + 2, ... into its three A slots; warp 8 streams the codes; lane 0 of
-// warps 9-12 (issuer e) issues the MMAs of units q = e, e + 4, ... into its own accumulator of
-// the job's buffer (two buffers, job parity); warps 13-16 and 17-20 are two epilogue groups
-// (job parity) that also build the B tiles of every call together.
+// decoding units q = s, s + 2, ... into A slot q % 12; warp 8 streams the codes; lane 0 of warps
+// 9-16 (issuer e) issues the MMAs of the units v = e, e + 8, ... of every job (counted from a
+// rotating start) into the job's accumulator (two buffers, job parity); warps 17-20 and 21-24 are
+// two epilogue groups (job parity) that also build the B tiles of every call together.
+// A thread blocks for about 150 cycles on each MMA it issues whatever the accumulator, so the
+// issue rate grows with the number of issuing warps; all of them add into one accumulator per
+// job (the digit sums are exact in f32, so their order does not matter), which the epilogue
+// reads and zeroes.
 #include <cuda.h>
 #include <cuda_bf16.h>
 
@@ -57,17 +61,18 @@ namespace ch {
 constexpr int kSets = 2;                 // decoder sets of four warps
 constexpr int kDecWarps = 4 * kSets;     // warps 0-7
 constexpr int kCopyWarp = kDecWarps;     // 8
-constexpr int kIss = 4;                  // MMA-issuing threads
-constexpr int kIssWarp0 = kCopyWarp + 1; // 9-12
-constexpr int kEpiWarp0 = kIssWarp0 + kIss;   // 13-20: two groups of four
+constexpr int kIss = 8;                  // MMA-issuing threads
+constexpr int kIssWarp0 = kCopyWarp + 1; // 9-16
+constexpr int kEpiWarp0 = kIssWarp0 + kIss;   // 17-24: two groups of four
 constexpr int kBThreads = 256;           // the two epilogue groups build the B tiles
 constexpr int kWarps = kEpiWarp0 + 8;
 constexpr int kThreads = kWarps * 32;
-constexpr int kSlots = 3;                // A slots per decoder set
+constexpr int kSlots = 12;               // A slots (unit q in slot q % kSlots)
+constexpr int kSetSlots = kSlots / kSets;
 constexpr int kDigits = 14;
 constexpr int kN = 32;                   // MMA N (2 kDigits used)
-constexpr int kColAcc = 0;               // accumulators [buffer][issuer], 32 columns each
-constexpr int kColA = 256;               // A slots [set][slot], 32 columns each
+constexpr int kColAcc = 0;               // accumulators [buffer], 32 columns each
+constexpr int kColA = 64;                // A slots, 32 columns each
 constexpr int kColSF = 448;              // unit scale factors
 constexpr int kTmemCols = 512;
 constexpr int kSlotCols = 32;
@@ -83,6 +88,7 @@ constexpr int kSmemLimit = 227 * 1024;
 constexpr uint64_t kWaitNs = 1000000000ull;   // 1 s: a pipeline wait is microseconds
 constexpr uint32_t kIdesc = idesc_mxf4_f32(128, kN);
 constexpr int kBarB = 1, kBarG = 2;      // named barriers: B build (256), epilogue group g (128)
+constexpr int kFixedBars = 2 * kSlots + 8 + kIss + 1;   // mbarriers besides the ring's
 
 struct Call {
   const void* x;
@@ -138,7 +144,7 @@ __host__ __device__ inline Smem smem_layout(int nring, int nu_max, int ncalls) {
   s.outp = s.gather + 2 * kMaxCluster * 64 * 4;
   s.tab = s.outp + 2 * 64 * 4;
   s.bar = s.tab + ncalls * (int)sizeof(Tab);
-  s.misc = s.bar + (2 * nring + 25) * 8;
+  s.misc = s.bar + (2 * nring + kFixedBars) * 8;
   s.total = s.misc + (int)sizeof(Misc) + 1024;   // + alignment slack
   return s;
 }
@@ -282,6 +288,16 @@ __device__ __forceinline__ void tmem_ld4(uint32_t taddr, float* v) {
   for (int i = 0; i < 4; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// Zeroes 16 columns of the warp's 32 TMEM lanes.
+__device__ __forceinline__ void tmem_zero16(uint32_t taddr) {
+  const uint32_t z = 0u;
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %1, %1, %1, %1, %1, %1, %1, %1, %1, %1, "
+      "%1, %1, %1, %1, %1};" ::"r"(taddr),
+      "r"(z)
+      : "memory");
+}
+
 // Bounded wait until *counter >= target (acquire); gives up early once any CTA has latched a
 // timeout in the status word.
 __device__ bool wait_counter(const unsigned int* counter, unsigned int target, volatile int* abort,
@@ -358,9 +374,9 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L.bar);
   uint64_t* full = bars;                       // [ring slot] codes landed (tx)
   uint64_t* empty = full + nring;              // [ring slot] codes read (4 warps)
-  uint64_t* sfull = empty + nring;             // [set][slot] A written (4 warps)
-  uint64_t* sfree = sfull + kSets * kSlots;    // [set][slot] its MMAs done (1 commit)
-  uint64_t* jfull = sfree + kSets * kSlots;    // [buffer] job accumulated (4 issuers)
+  uint64_t* sfull = empty + nring;             // [slot] A written (4 warps)
+  uint64_t* sfree = sfull + kSlots;            // [slot] its MMAs done (1 commit)
+  uint64_t* jfull = sfree + kSlots;            // [buffer] job accumulated (every issuer)
   uint64_t* jfree = jfull + 2;                 // [buffer] job read out (4 warps)
   uint64_t* gfull = jfree + 2;                 // [group] rank 0: partials arrived (tx)
   uint64_t* gfree = gfull + 2;                 // [group] ranks > 0: rank 0 read the buffer (1)
@@ -391,12 +407,12 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
     tab[c] = t;
   }
   if (warp == 1) {
-    const int nb = 2 * nring + 25;
+    const int nb = 2 * nring + kFixedBars;
     for (int i = lane; i < nb; i += 32) {
       uint64_t* b = bars + i;
       uint32_t cnt = 1;
       if (b >= empty && b < empty + nring) cnt = 4;
-      else if (b >= sfull && b < sfull + kSets * kSlots) cnt = 4;
+      else if (b >= sfull && b < sfull + kSlots) cnt = 4;
       else if (b == jfull || b == jfull + 1) cnt = kIss;
       else if (b == jfree || b == jfree + 1) cnt = 4;
       else if (b == sfready) cnt = 4;
@@ -419,13 +435,18 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
     NJ += tab[c].nj;
   }
   if (warp < 4) {
-    // Unit scale factors (ue8m0 127 = 1.0) for every row of A and B of every MMA.
+    // Unit scale factors (ue8m0 127 = 1.0) for every row of A and B of every MMA; both
+    // accumulators start at zero (every MMA adds).
     uint32_t ones[32];
 #pragma unroll
     for (int i = 0; i < 32; ++i) ones[i] = 0x7F7F7F7Fu;
-    const uint32_t la = tmem + ((uint32_t)(warp * 32) << 16) + kColSF;
-    tmem_st32(la, ones);
-    tmem_st32(la + 32, ones);
+    const uint32_t la = tmem + ((uint32_t)(warp * 32) << 16);
+    tmem_st32(la + kColSF, ones);
+    tmem_st32(la + kColSF + 32, ones);
+#pragma unroll
+    for (int i = 0; i < 32; ++i) ones[i] = 0u;
+    tmem_st32(la + kColAcc, ones);
+    tmem_st32(la + kColAcc + 32, ones);
     tmem_wait_st();
     tc_fence_before();
     __syncwarp();
@@ -452,7 +473,7 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
     const uint32_t h0 = ((lane >> 2) & 1u) * 16u;   // which 16-byte half first (bank spread)
     const uint32_t ring = smem_u32(smem + L.ring);
     const uint32_t t_lane = tmem + ((uint32_t)(quarter * 32) << 16) + kColA;
-    int rs = set, sl = 0, l = 0;
+    int rs = set, si = set, l = 0;   // ring slot, A slot, units of this set so far
     uint32_t rph = 0, sph = 0;
     if (rs >= nring) { rs -= nring; rph ^= 1u; }
     for (int q = set; q < Q; q += kSets, ++l) {
@@ -467,7 +488,7 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
       v[3] = lds128(src + chunk1 + (16u - h0));
       __syncwarp();
       if (lane == 0) mbar_arrive(&empty[rs]);
-      if (l == kSlots) pdl_wait_primary();   // later waits depend on MMAs, i.e. on x
+      if (l == kSetSlots) pdl_wait_primary();   // later waits depend on MMAs, i.e. on x
       const uint4 a0 = h0 ? v[1] : v[0], a1 = h0 ? v[0] : v[1];
       const uint4 b0 = h0 ? v[3] : v[2], b1 = h0 ? v[2] : v[3];
       const uint32_t w0[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
@@ -476,8 +497,7 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
       decode_chunk(w0, sel, rr);
       decode_chunk(w1, sel, rr + 16);
       // the slot's previous unit has been multiplied (only the store waits for it)
-      const int si = set * kSlots + sl;
-      if (l >= kSlots) {
+      if (l >= kSetSlots) {
         if (!__all_sync(0xffffffffu, mbar_test_wait(&sfree[si], sph ^ 1u) ||
                                          spin_or_abort(&sfree[si], sph ^ 1u, abort_flag, a.status)))
           break;
@@ -488,8 +508,9 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&sfull[si]);
-      if (++sl == kSlots) {
-        sl = 0;
+      si += kSets;
+      if (si >= kSlots) {
+        si -= kSlots;
         sph ^= 1u;
       }
       rs += kSets;
@@ -568,34 +589,37 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
         (void)mbar_wait_timed(&full[i % nring], (i / nring) & 1, 1000000ull);
     }
   } else if (warp < kEpiWarp0) {
-    // ---- MMA issuers: lane 0 of warp kIssWarp0 + e issues units q = e, e + 4, ... ----
-    const int e = warp - kIssWarp0, set = e & 1;
+    // ---- MMA issuers: lane 0 of warp kIssWarp0 + e issues unit v of a job when
+    // (v + r) % kIss == e, r = the units of this CTA before the job; unit q (counted over the
+    // whole chain) sits in A slot q % kSlots ----
+    const int e = warp - kIssWarp0;
     if (lane == 0) {
       const uint32_t b_base = smem_u32(smem + L.b);
       const uint64_t desc0 = smem_desc(b_base, 128, 256);
       pdl_wait_primary();
       bool ok = wait_or_abort(sfready, 0, abort_flag, a.status);
       bool issued = false;
-      int sl = e >> 1, J = 0, q4 = 0;
-      uint32_t sph = 0, seq = 0;
+      int J = 0, qb = 0;   // jobs and units before the current job
+      uint32_t seq = 0;
       for (int c = 0; ok && c < ncalls; ++c) {
         const Tab tb = tab[c];
         if (tb.nj == 0) continue;
         const int U = (tb.nu + 1) >> 1;
         ++seq;   // this call's B tiles are the seq-th build; unit v needs its chunks built
         int have = 0;
-        for (int k = 0; ok && k < tb.nj; ++k, ++J) {
+        for (int k = 0; ok && k < tb.nj; ++k, ++J, qb += U) {
           const int buf = J & 1;
-          // the read-out of job J - 2 (same buffer) is done
+          // the read-out of job J - 2 (same buffer) is done and the accumulator zeroed
           if (J >= 2) ok = wait_or_abort(&jfree[buf], ((J >> 1) - 1) & 1, abort_flag, a.status);
           if (!ok) break;
           tc_fence_after();
-          const int v0 = (e - q4) & 3;
+          const int v0 = (e - qb) & (kIss - 1);
           if (v0 < U) {
-            const uint32_t d_tmem = tmem + kColAcc + (uint32_t)((buf * kIss + e) * 32);
-            bool first = true;
-            for (int v = v0; v < U; v += 4) {
-              const int si = set * kSlots + sl;
+            const uint32_t d_tmem = tmem + kColAcc + (uint32_t)(buf * 32);
+            const int q0 = qb + v0;
+            int si = q0 % kSlots;
+            uint32_t sph = (uint32_t)(q0 / kSlots) & 1u;
+            for (int v = v0; v < U; v += kIss) {
               const int need = min(tb.nu, 2 * v + 2);
               if (have < need) {
                 ok = wait_bprog(&misc->bprog, (seq << 8) | (uint32_t)need, abort_flag, a.status);
@@ -613,13 +637,12 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
               for (int jm = 0; jm < 4; ++jm)
                 if (jm < nm)
                   mma_mxf4_ts(d_tmem, a_slot + jm * 8, bd + (uint64_t)((jm * kMmaB) >> 4), kIdesc,
-                              tmem + kColSF, tmem + kColSF + 16, (first && jm == 0) ? 0u : 1u);
-              first = false;
+                              tmem + kColSF, tmem + kColSF + 16, 1u);
               issued = true;
               mma_commit(&sfree[si]);
-              sl += 2;
-              if (sl >= kSlots) {
-                sl -= kSlots;
+              si += kIss;   // this issuer's next unit: q + kIss (kIss < kSlots)
+              if (si >= kSlots) {
+                si -= kSlots;
                 sph ^= 1u;
               }
             }
@@ -628,7 +651,6 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
           } else {
             mbar_arrive(&jfull[buf]);
           }
-          q4 = (q4 + U) & 3;
         }
       }
       // Abort path: the MMAs this thread issued finish before TMEM is released.
@@ -653,7 +675,7 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
     }
     pdl_wait_primary();   // x may be written, and y read, by the previous kernel
     if (ks > 1) cluster_wait();   // every rank's barriers are initialised
-    int nbuilt = 0, J = 0, q4 = 0;
+    int nbuilt = 0, J = 0;
     for (int c = 0; c < ncalls; ++c) {
       const Tab tb = tab[c];
       const Call& C = a.calls[c];
@@ -787,7 +809,6 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
         }
         ++nbuilt;
         const float invS = misc->invS;
-        const int U = (tb.nu + 1) >> 1;
 
         // -------- the jobs of call c: group grp reads out the jobs of its parity --------
         int g = tb.first / C.rbs, rb = tb.first - g * C.rbs;
@@ -799,25 +820,24 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
             tc_fence_after();
             float vre = 0.f, vim = 0.f;
             if (got) {
-              const uint32_t acc0 = tmem + ((uint32_t)(quarter * 32) << 16) + kColAcc +
-                                    (uint32_t)(grp * kIss * 32);
-              // one issuer's 28 digit columns per round (loads of 16 + 8 + 4, one wait)
-#pragma unroll 1
-              for (int e = 0; e < kIss; ++e) {
-                if (((e - q4) & 3) >= U) continue;
-                float d[28];
-                const uint32_t ta = acc0 + e * 32;
-                tmem_ld16(ta, *reinterpret_cast<float(*)[16]>(&d[0]));
-                tmem_ld8(ta + 16, &d[16]);
-                tmem_ld4(ta + 24, &d[24]);
-                tmem_wait_ld();
+              // the 28 digit columns (loads of 16 + 8 + 4, one wait), then zeroes for the
+              // job after next
+              const uint32_t ta = tmem + ((uint32_t)(quarter * 32) << 16) + kColAcc +
+                                  (uint32_t)(grp * 32);
+              float d[28];
+              tmem_ld16(ta, *reinterpret_cast<float(*)[16]>(&d[0]));
+              tmem_ld8(ta + 16, &d[16]);
+              tmem_ld4(ta + 24, &d[24]);
+              tmem_wait_ld();
 #pragma unroll
-                for (int l = 0; l < kDigits; ++l) {
-                  const float wgt = (float)(1u << (2 * l));
-                  vre = fmaf(d[l], wgt, vre);
-                  vim = fmaf(d[kDigits + l], wgt, vim);
-                }
+              for (int l = 0; l < kDigits; ++l) {
+                const float wgt = (float)(1u << (2 * l));
+                vre = fmaf(d[l], wgt, vre);
+                vim = fmaf(d[kDigits + l], wgt, vim);
               }
+              tmem_zero16(ta);
+              tmem_zero16(ta + 16);
+              tmem_wait_st();
             }
             tc_fence_before();
             __syncwarp();
@@ -896,7 +916,6 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
               }
             }
           }
-          q4 = (q4 + U) & 3;
           rb += ncl;
           while (rb >= C.rbs) {
             rb -= C.rbs;
