@@ -1,20 +1,30 @@
 """Benchmark of the quantized widely-linear layer on a LLaMA-2-7B-shaped linear stack.
 
-Workload (default): 32 decoder layers x {q, k, v, o, gate, up, down} (hidden 4096, intermediate
+Workload (headline): 32 decoder layers x {q, k, v, o, gate, up, down} (hidden 4096, intermediate
 11008), every weight Student-t(df=4, std 0.02), converted and quantized with T=2 stages; one
 step = one decode token (batch 1, bf16 activations with 1% outlier channels) through all 224
 quantized linears, as a decoder layer feeds them: q, k, v on one input (one grouped call), o,
-gate and up on one input (one grouped call), down; 4 calls per layer (--ungrouped: 7). Metric: decode GB/s = algorithmic bytes (packed codes + scales + x + y of
-every linear) per second, against the HBM copy peak. The 1.62 GB of codes per step exceed the
-L2 many times over, so no L2 flush is needed between steps.
+gate and up on one input (one grouped call), down; 4 calls per layer (--ungrouped: 7). Metric:
+decode GB/s = algorithmic bytes (packed codes + scales + x + y of every linear) per second,
+against the HBM copy peak. The 1.62 GB of codes per step exceed the L2 many times over, so no
+L2 flush is needed between steps.
 
-The line also carries a "prefill" object: the tensor-core GEMM path on 2048 tokens through the
-4096 -> 11008 and 11008 -> 4096 layers at T = 1, 2, 3 (effective TOPS = 8 n m B / time, and the
-MMA work 16 T n m B / time against the bf16 tensor peak), each launch timed alone with CUDA
-events after an L2 flush.
+Further objects on the same line (each timed with CUDA events on the launching stream):
+* decode_chain: the same step as one persistent launch (fairy2i_wl_matmul_chain, 128 calls,
+  call c reading its input only after call c - 1's outputs are written);
+* batches: the stack at batch 8 and 64 (per-token time), the MLP layers (gate, up, down) at
+  batch 1, 4 and 16 and the attention projections (4096 -> 4096) at batch 1, each over all 32
+  layers' weights so that the codes come from HBM;
+* quantize: convert and quantize of the 4096 -> 11008 layer (T = 1, 2, 3), GB/s;
+* prefill: the tensor-core GEMM path on 2048 tokens through the 4096 -> 11008 and
+  11008 -> 4096 layers at T = 1, 2, 3 (effective TOPS = 8 n m B / time, and the MMA work
+  16 T n m B / time against the bf16 tensor peak), each launch timed alone after an L2 flush;
+* lut_cpu: the look-up-table matmul on the host cores (one 4096 -> 4096 linear, one token);
+* cpu_baseline: the float64 oracle on the host cores (all cores, and one thread) on a bounded
+  sample (layer 0's q and k at the headline batch).
 
---impl reference times the CPU oracle (float64 numpy) on the host cores on a bounded sample of
-the same workload and reports the same metric.
+--impl reference times the CPU oracle on the host cores on the same sample as cpu_baseline and
+reports the same metric.
 
 Multi-GPU: the layer is not partitioned across ranks; N ranks run N independent replicas
 (weak scaling) and value = bytes of all ranks / max over ranks of the timed region.
@@ -41,6 +51,8 @@ from paper_2512_02901_gb300 import synth  # noqa: E402
 METRIC = "WL {±1,±i} matmul: decode GB/s vs HBM peak; prefill effective TOPS"
 WORKLOAD = "llama2-7b-linear-stack-decode"
 T_STAGES = 2
+HBM_NOMINAL_GBS = 7900.0
+SAMPLE_LINEARS = 2   # layer 0's first linears (q, k) timed by cpu_baseline and --impl reference
 
 
 def peaks():
@@ -56,34 +68,36 @@ def peaks():
 # current kernels: one decoder layer's decode launches (every layer has the same shapes; grouped:
 # q/k/v, o, gate/up, down; ungrouped: seven), and one T = 2 prefill launch of the 4096 -> 11008
 # layer on 2048 tokens. Per call and decode kernel: "fp8" = the warp-MMA kernel, "stream" = the
-# persistent tcgen05 kernel (grouped calls: q/k/v, gate/up).
+# persistent tcgen05 kernel's one-token form.
 DECODE_DRAM_BYTES = {
     "fp8": {"q,k,v": 12.621e6, "o": 4.232e6, "gate,up": 22.582e6, "down": 11.323e6,
             "q": 4.231e6, "k": 4.231e6, "v": 4.231e6, "gate": 11.309e6, "up": 11.309e6},
-    "stream": {"q,k,v": 12.666e6, "gate,up": 22.628e6},
+    "stream": {"q,k,v": 12.667e6, "o": 4.277e6, "gate,up": 22.628e6, "down": 11.369e6},
 }
 PREFILL_T2_UP_DRAM_BYTES = 28.089e6 + 36.948e6
+# ncu sm__pipe_tensor_cycles_active of the same prefill launch (T = 2, up layer, 2048 tokens)
+PREFILL_T2_UP_TENSOR_PIPE_PCT = 52.7
+
 
 def decode_kernel(c, path, sms):
-    """The decode kernel the library runs for a call at batch <= 2: the automatic path takes the
-    persistent tcgen05 kernel when the call's 16-row tiles outnumber the SMs."""
+    """The decode kernel the library runs for a call at batch <= 2 (bf16 x): the automatic path
+    takes the persistent tcgen05 kernel's one-token form, token by token."""
     if path == 1:
         return "fp8"
-    if path == 4:
-        return "stream"
-    n = (c["rows"] + 1) // 2
-    return "stream" if len(c["members"]) * ((n + 15) // 16) > sms else "fp8"
+    if path == 5:
+        return "chain"
+    return "stream"
 
 
-def decode_traffic(calls, args, sms):
+def decode_traffic(calls, path, B, sms):
     """ncu DRAM bytes of one step's decode launches (batch 1), summed per call from captures of
     the kernels this run uses; None where no capture exists for a call."""
-    if args.batch != 1:
+    if B != 1:
         return None
     total = 0.0
     for c in calls:
         name = ",".join(m["name"] for m in c["members"])
-        v = DECODE_DRAM_BYTES[decode_kernel(c, args.decode_path, sms)].get(name)
+        v = DECODE_DRAM_BYTES[decode_kernel(c, path, sms)].get(name)
         if v is None:
             return None
         total += v
@@ -193,20 +207,9 @@ def max_over_ranks(v: float, world: int) -> float:
 GROUPS = (("q", "k", "v"), ("o",), ("gate", "up"), ("down",))   # linears sharing an input
 
 
-def build_stack(F, layers: int, B: int, dev, grouped: bool = True):
-    """Converts + quantizes every linear of the stack on the GPU; returns the calls of a step:
-    per call the input x and its member linears (one member each when not grouped). The inputs
-    of all calls are views of one buffer, the outputs of another, so that a step's activations
-    reach the device and its results the host in one copy each."""
-    groups = GROUPS if grouped else tuple((nm,) for g in GROUPS for nm in g)
-    cols_of = {name: cols for (_, _, name, _, cols) in layer_shapes(1)}
-    rows_of = {name: rows for (_, _, name, rows, _) in layer_shapes(1)}
-    x_all = torch.empty(layers * sum(B * cols_of[g[0]] for g in groups), dtype=torch.bfloat16,
-                        device=dev)
-    y_all = torch.empty(layers * sum(B * rows_of[nm] for g in groups for nm in g),
-                        dtype=torch.float32, device=dev)
-    xo = yo = 0
-    calls = []
+def build_linears(F, layers: int, dev):
+    """Converts + quantizes every linear of the stack on the GPU: [layer][name] -> dict."""
+    out = []
     for L in range(layers):
         lin = {}
         for (_, pi, name, rows, cols) in layer_shapes(1):
@@ -218,21 +221,40 @@ def build_stack(F, layers: int, B: int, dev, grouped: bool = True):
             del U, W
             lin[name] = dict(L=L, name=name, seed=seed, rows=rows, cols=cols, codes=codes,
                              scales=scales)
-        for g in groups:
-            first = lin[g[0]]
-            for nm in g:
-                lin[nm]["y"] = y_all[yo:yo + B * lin[nm]["rows"]].view(B, lin[nm]["rows"])
-                yo += B * lin[nm]["rows"]
-            x = x_all[xo:xo + B * first["cols"]].view(B, first["cols"])
-            xo += B * first["cols"]
-            x.copy_(synth.outlier_activations(B, first["cols"],
-                                              synth.activation_seed(first["seed"], B), device=dev))
-            calls.append(dict(x=x, rows=first["rows"], cols=first["cols"],
-                              members=[lin[nm] for nm in g]))
+        out.append(lin)
     torch.cuda.synchronize()
     status = F.get_status()
     if status != 0:
         raise RuntimeError(f"quantize status {status}")
+    return out
+
+
+def make_calls(linears, B: int, dev, groups=GROUPS):
+    """The calls of a step over `linears` at batch B: per call the input x and its member
+    linears with their outputs. The inputs of all calls are views of one buffer, the outputs of
+    another, so that a step's activations reach the device and its results the host in one copy
+    each."""
+    cols_of = {name: cols for (_, _, name, _, cols) in layer_shapes(1)}
+    rows_of = {name: rows for (_, _, name, rows, _) in layer_shapes(1)}
+    x_all = torch.empty(len(linears) * sum(B * cols_of[g[0]] for g in groups),
+                        dtype=torch.bfloat16, device=dev)
+    y_all = torch.empty(len(linears) * sum(B * rows_of[nm] for g in groups for nm in g),
+                        dtype=torch.float32, device=dev)
+    xo = yo = 0
+    calls = []
+    for lin in linears:
+        for g in groups:
+            first = lin[g[0]]
+            ys = []
+            for nm in g:
+                ys.append(y_all[yo:yo + B * rows_of[nm]].view(B, rows_of[nm]))
+                yo += B * rows_of[nm]
+            x = x_all[xo:xo + B * first["cols"]].view(B, first["cols"])
+            xo += B * first["cols"]
+            x.copy_(synth.outlier_activations(B, first["cols"],
+                                              synth.activation_seed(first["seed"], B), device=dev))
+            calls.append(dict(x=x, rows=first["rows"], cols=first["cols"], ys=ys,
+                              members=[lin[nm] for nm in g]))
     return calls, x_all, y_all
 
 
@@ -242,14 +264,44 @@ def call_bytes(c, B):
     return sum(per) - (len(per) - 1) * B * c["cols"] * 2
 
 
-def run_call(F, c, path=0):
+def run_call(F, c, path=0, stream=None):
     if len(c["members"]) == 1:
         m = c["members"][0]
-        F.wl_matmul(c["x"], m["codes"], m["scales"], c["rows"], y=m["y"], path=path)
+        F.wl_matmul(c["x"], m["codes"], m["scales"], c["rows"], y=c["ys"][0], path=path,
+                    stream=stream)
     else:
         F.wl_matmul_group(c["x"], [m["codes"] for m in c["members"]],
-                          [m["scales"] for m in c["members"]], c["rows"],
-                          ys=[m["y"] for m in c["members"]], path=path)
+                          [m["scales"] for m in c["members"]], c["rows"], ys=c["ys"], path=path,
+                          stream=stream)
+
+
+def graphed(fn, stream, warmup: int):
+    """fn captured once in a CUDA graph on `stream` (after `warmup` eager runs); returns the
+    replay."""
+    with torch.cuda.stream(stream):
+        for _ in range(max(warmup, 1)):
+            fn()
+    stream.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        fn()
+    stream.synchronize()
+    return g.replay
+
+
+def time_replays(run, stream, reps: int, warmup: int = 3) -> float:
+    """Milliseconds per run() over `reps` runs (CUDA events on `stream`)."""
+    with torch.cuda.stream(stream):
+        for _ in range(warmup):
+            run()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            run()
+        e1.record(stream)
+    stream.synchronize()
+    return e0.elapsed_time(e1) / reps
 
 
 def run_ours(args, world, rank, local):
@@ -259,7 +311,9 @@ def run_ours(args, world, rank, local):
     F.load()
     dev = torch.device("cuda", local)
     B = args.batch
-    calls, x_all, y_all = build_stack(F, args.layers, B, dev, grouped=not args.ungrouped)
+    groups = GROUPS if not args.ungrouped else tuple((nm,) for g in GROUPS for nm in g)
+    linears = build_linears(F, args.layers, dev)
+    calls, x_all, y_all = make_calls(linears, B, dev, groups)
     step_bytes = sum(call_bytes(c, B) for c in calls)
     nlinears = sum(len(c["members"]) for c in calls)
     # a grouped call is one launch where the decode kernel takes it (B <= 2), else one per member
@@ -270,18 +324,7 @@ def run_ours(args, world, rank, local):
             run_call(F, c, args.decode_path)
 
     stream = torch.cuda.Stream(device=dev)
-    with torch.cuda.stream(stream):
-        for _ in range(max(args.warmup, 1)):
-            step()
-    stream.synchronize()
-    graph = None
-    if not args.no_graph:
-        graph = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(graph, stream=stream):
-            step()
-        stream.synchronize()
-    run = (lambda: graph.replay()) if graph is not None else step
-
+    run = step if args.no_graph else graphed(step, stream, args.warmup)
     with torch.cuda.stream(stream):
         for _ in range(args.warmup):
             run()
@@ -293,6 +336,14 @@ def run_ours(args, world, rank, local):
     barrier(world)
     torch.cuda.synchronize()
     clocks.start()
+    # the sampler sees the GPU under load for ~0.3 s before the timed region as well
+    t_end = time.perf_counter() + 0.3
+    with torch.cuda.stream(stream):
+        while time.perf_counter() < t_end:
+            run()
+            stream.synchronize()
+    barrier(world)
+    torch.cuda.synchronize()
     with torch.cuda.stream(stream):
         e0.record(stream)
         for _ in range(args.steps):
@@ -323,21 +374,10 @@ def run_ours(args, world, rank, local):
         run()
         y_host.copy_(y_all, non_blocking=True)
 
-    with torch.cuda.stream(stream):
-        for _ in range(args.warmup):
-            e2e_step()
-    stream.synchronize()
-    e2 = torch.cuda.Event(enable_timing=True)
-    e3 = torch.cuda.Event(enable_timing=True)
     e2e_steps = max(1, min(args.steps, 50))
     barrier(world)
-    with torch.cuda.stream(stream):
-        e2.record(stream)
-        for _ in range(e2e_steps):
-            e2e_step()
-        e3.record(stream)
-    stream.synchronize()
-    ms_e2e = max_over_ranks(e2.elapsed_time(e3), world)
+    ms_e2e = max_over_ranks(time_replays(e2e_step, stream, e2e_steps, args.warmup) * e2e_steps,
+                            world)
     st = F.get_status()
     if st != 0:
         raise RuntimeError(f"device status {st} after the end-to-end steps")
@@ -346,8 +386,12 @@ def run_ours(args, world, rank, local):
     hbm, _, peak_kind = peaks()
     achieved = step_bytes / (ms_step * 1e-3) / 1e9
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
-    traffic = decode_traffic(calls, args, sms)
+    traffic = decode_traffic(calls, args.decode_path, B, sms)
     kernels = sorted({decode_kernel(c, args.decode_path, sms) for c in calls}) if B <= 2 else []
+    kname = ("wl_matmul decode (all launches of the step: "
+             + " + ".join({"fp8": "warp-MMA", "stream": "persistent tcgen05",
+                           "chain": "chained tcgen05"}[k] for k in kernels)
+             + ")") if kernels else "wl_matmul (all launches of the step: tcgen05 GEMM)"
     line = {
         "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_step, 5),
@@ -359,7 +403,7 @@ def run_ours(args, world, rank, local):
                    "grouping": "none" if args.ungrouped else "qkv, o, gate+up, down (shared x)",
                    "decode_path": args.decode_path,
                    "T": T_STAGES, "batch": B, "x_dtype": "bf16",
-                   "bytes_per_step": step_bytes, "cuda_graph": graph is not None,
+                   "bytes_per_step": step_bytes, "cuda_graph": not args.no_graph,
                    "l2": "inputs larger than L2 (packed codes per step >> 129 MB)",
                    "parallelism": f"replicas{world}"},
         "e2e": {"value": round(e2e_value, 2), "unit": "GB/s", "h2d_bytes_per_step": h2d,
@@ -367,20 +411,152 @@ def run_ours(args, world, rank, local):
         "gpu_launches": launches_per_step * args.steps,
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm,
                      "unit": "GB/s", "frac": round(achieved / hbm, 4),
+                     "frac_nominal": round(achieved / HBM_NOMINAL_GBS, 4),
                      "traffic": traffic,
-                     "peak_kind": f"{peak_kind} hbm_gbs (burst copy)",
-                     "kernel": "wl_matmul decode (all launches of the step: "
-                               + " + ".join({"fp8": "warp-MMA", "stream": "persistent tcgen05"}[k]
-                                            for k in kernels) + ")"},
+                     "peak_kind": f"{peak_kind} hbm_gbs (burst copy); frac_nominal against "
+                                  f"{HBM_NOMINAL_GBS:.0f} GB/s nominal",
+                     "kernel": kname},
         "clocks": clk,
     }
+    del x_host, y_host
+    if B == 1 and not args.ungrouped and not args.no_chain:
+        line["decode_chain"] = run_chain(F, calls, dev, step_bytes, args)
+    del calls, x_all, y_all
+    torch.cuda.empty_cache()
+    if not args.no_sweep:
+        line["batches"] = run_batches(F, linears, dev, args)
+    del linears
+    torch.cuda.empty_cache()
+    if not args.no_quantize:
+        line["quantize"] = run_quantize(F, dev)
     if not args.no_prefill:
-        del calls, x_all, y_all
-        torch.cuda.empty_cache()
         line["prefill"] = run_prefill(F, dev, args.prefill_steps, max(args.warmup, 3))
+    if rank == 0 and not args.no_lut:
+        line["lut_cpu"] = run_lut(F)
     if rank == 0 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(B, budget_s=args.cpu_budget)
+        line["cpu_baseline"] = cpu_baseline(B, budget_s=args.cpu_budget, count=args.ref_linears)
     return line
+
+
+def run_chain(F, calls, dev, step_bytes, args):
+    """The step as one launch of the chained decode kernel."""
+    hbm, _, peak_kind = peaks()
+    tup = [(c["x"], [m["codes"] for m in c["members"]], [m["scales"] for m in c["members"]],
+            c["ys"], c["rows"]) for c in calls]
+    arr = F.chain_calls(tup)
+    ws = F.chain_workspace(len(tup), dev)
+    stream = torch.cuda.Stream(device=dev)
+    run = graphed(lambda: F.wl_matmul_chain(None, T_STAGES, workspace=ws, stream=stream, arr=arr),
+                  stream, 2)
+    reps = max(5, min(args.steps, 50))
+    ms = time_replays(run, stream, reps, max(args.warmup, 3))
+    if F.get_status() != 0:
+        raise RuntimeError("device status after the chained decode")
+    gbs = step_bytes / (ms * 1e-3) / 1e9
+    return {"workload": f"{WORKLOAD} (batch 1), one launch", "calls": len(tup),
+            "us_per_step": round(ms * 1e3, 1), "value": round(gbs, 1), "unit": "GB/s",
+            "frac": round(gbs / hbm, 4), "frac_nominal": round(gbs / HBM_NOMINAL_GBS, 4),
+            "peak_kind": f"{peak_kind} hbm_gbs", "gpu_launches": reps}
+
+
+def run_batches(F, linears, dev, args):
+    """Other batches: the whole stack at batch 8 and 64 (per token), the MLP layers at batch 1,
+    4 and 16, the attention projections at batch 1; every figure runs over all layers' weights
+    (codes from HBM), through the automatic path."""
+    hbm, _, _ = peaks()
+    stream = torch.cuda.Stream(device=dev)
+    out = []
+    cases = [("stack", GROUPS, 8), ("stack", GROUPS, 64),
+             ("mlp gate+up, down", (("gate", "up"), ("down",)), 1),
+             ("mlp gate+up, down", (("gate", "up"), ("down",)), 4),
+             ("mlp gate+up, down", (("gate", "up"), ("down",)), 16),
+             ("attention q, k, v, o (4096->4096 each)", (("q",), ("k",), ("v",), ("o",)), 1)]
+    for name, groups, B in cases:
+        calls, x_all, y_all = make_calls(linears, B, dev, groups)
+        nbytes = sum(call_bytes(c, B) for c in calls)
+        nlin = sum(len(c["members"]) for c in calls)
+
+        def step():
+            for c in calls:
+                run_call(F, c, 0, stream)
+
+        run = graphed(step, stream, 1)
+        reps = 5 if B >= 16 else 10
+        ms = time_replays(run, stream, reps, 2)
+        if F.get_status() != 0:
+            raise RuntimeError(f"device status after batch {B} ({name})")
+        gbs = nbytes / (ms * 1e-3) / 1e9
+        rec = {"case": name, "batch": B, "layers": len(linears), "linears": nlin,
+               "us_per_pass": round(ms * 1e3, 1), "value": round(gbs, 1), "unit": "GB/s",
+               "frac": round(gbs / hbm, 4)}
+        if name == "stack":
+            rec["us_per_token"] = round(ms * 1e3 / B, 2)
+        if name.startswith("attention"):
+            rec["us_per_linear"] = round(ms * 1e3 / nlin, 2)
+        if name.startswith("mlp"):
+            rec["us_per_layer"] = round(ms * 1e3 / len(linears), 2)
+        rec["path"] = "decode kernels" if B <= 2 else "tcgen05 GEMM (64-token tiles)"
+        out.append(rec)
+        del calls, x_all, y_all
+    torch.cuda.empty_cache()
+    return out
+
+
+def run_quantize(F, dev):
+    """convert + quantize of the 4096 -> 11008 layer: median of 5 timed runs each (L2 flushed
+    before each), GB/s of the traffic each makes: convert reads R and writes U, W; quantize reads
+    U, W T + 1 times (T stage passes and the pack pass) and writes the codes."""
+    hbm, _, _ = peaks()
+    rows, cols = 11008, 4096
+    n, m = (rows + 1) // 2, (cols + 1) // 2
+    R = synth.student_t_weight(rows, cols, synth.weight_seed("prefill", 0), device=dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.Stream(device=dev)
+    stream.wait_stream(torch.cuda.current_stream())
+
+    def timed(fn, reps=5):
+        ts = []
+        with torch.cuda.stream(stream):
+            for i in range(reps + 2):
+                flush.zero_()
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                fn()
+                e1.record(stream)
+                if i >= 2:
+                    ts.append((e0, e1))
+        stream.synchronize()
+        return statistics.median(a.elapsed_time(b) for a, b in ts)
+
+    res = {}
+    U, W = F.convert(R, stream=stream)
+    ms_c = timed(lambda: F.convert(R, stream=stream))
+    conv_bytes = rows * cols * 4 + 2 * n * m * 8
+    res["convert"] = {"us": round(ms_c * 1e3, 1), "bytes": conv_bytes,
+                      "gbs": round(conv_bytes / (ms_c * 1e-3) / 1e9, 1),
+                      "frac": round(conv_bytes / (ms_c * 1e-3) / 1e9 / hbm, 4)}
+    res["quantize"] = []
+    for T in (1, 2, 3):
+        ws = torch.empty(F.quantize_workspace_bytes(n, m, T), dtype=torch.uint8, device=dev)
+        codes, scales = F.quantize(U, W, T, workspace=ws, stream=stream)
+        ms_q = timed(lambda: F.quantize(U, W, T, codes=codes, scales=scales, workspace=ws,
+                                        stream=stream))
+        code_bytes = T * 2 * n * m // 4
+        traffic = (T + 1) * 2 * n * m * 8 + code_bytes
+        once = 2 * n * m * 8 + code_bytes
+        res["quantize"].append({"T": T, "us": round(ms_q * 1e3, 1), "bytes": traffic,
+                                "gbs": round(traffic / (ms_q * 1e-3) / 1e9, 1),
+                                "frac": round(traffic / (ms_q * 1e-3) / 1e9 / hbm, 4),
+                                "one_read_gbs": round(once / (ms_q * 1e-3) / 1e9, 1)})
+        del codes, scales, ws
+    if F.get_status() != 0:
+        raise RuntimeError("device status after the quantize timing")
+    del R, U, W, flush
+    torch.cuda.empty_cache()
+    res["workload"] = f"{cols}->{rows} layer (complex {m}->{n}), fp32 weights"
+    res["timing"] = "median of 5 CUDA-event times, L2 flushed before each"
+    return res
 
 
 def run_prefill(F, dev, steps: int, warmup: int):
@@ -432,6 +608,7 @@ def run_prefill(F, dev, steps: int, warmup: int):
                 roof = {"bound": "tensor", "achieved": round(mma, 1), "peak": bf16,
                         "unit": "TFLOP/s", "frac": round(mma / bf16, 4),
                         "traffic": int(PREFILL_T2_UP_DRAM_BYTES),
+                        "ncu_tensor_pipe_active_pct": PREFILL_T2_UP_TENSOR_PIPE_PCT,
                         "peak_kind": f"{peak_kind} bf16_tflops (burst)",
                         "kernel": f"wl_prefill_kernel<{T}> (up {cols}->{rows}, "
                                   f"{PREFILL_TOKENS} tokens)"}
@@ -443,6 +620,36 @@ def run_prefill(F, dev, steps: int, warmup: int):
             "timing": "median of per-launch CUDA-event times, L2 flushed before each launch",
             "layers": rows_out, "roofline": roof, "clocks": clk,
             "gpu_launches": len(rows_out) * steps}
+
+
+def run_lut(F):
+    """The host look-up-table matmul (Sec. 3.4) on one 4096 -> 4096 linear (layer 0's q, codes
+    made by the GPU quantizer), one int8 token, all host cores and one."""
+    dev = torch.device("cuda", torch.cuda.current_device())
+    rows, cols = 4096, 4096
+    seed = synth.weight_seed("stack", 0, 0)
+    R = synth.student_t_weight(rows, cols, seed, device=dev)
+    U, W = F.convert(R)
+    codes, scales = F.quantize(U, W, T_STAGES)
+    codes, scales = codes.cpu(), scales.cpu()
+    del R, U, W
+    x = synth.outlier_activations(1, cols, synth.activation_seed(seed, 1)).float()
+    xq, delta = F.lut_quantize_x(x)
+    nb = layer_bytes(rows, cols, 1, x_bytes=1)
+    out = {"workload": "4096->4096 linear (complex 2048->2048), T = 2, one int8 token",
+           "unit": "GB/s (packed codes + scales + x + y)"}
+    for label, nt in (("all_cores", os.cpu_count() or 1), ("one_thread", 1)):
+        F.lut_matmul(xq, delta, codes, scales, rows, nthreads=nt)
+        reps, t0 = 0, time.perf_counter()
+        while True:
+            F.lut_matmul(xq, delta, codes, scales, rows, nthreads=nt)
+            reps += 1
+            if time.perf_counter() - t0 > 1.0 or reps >= 200:
+                break
+        sec = (time.perf_counter() - t0) / reps
+        out[label] = {"threads": nt, "us": round(sec * 1e6, 1),
+                      "value": round(nb / sec / 1e9, 3)}
+    return out
 
 
 # --------------------------------------------------------------------------------------------
@@ -460,42 +667,65 @@ def _threads():
         from threadpoolctl import threadpool_info
         return max(int(i.get("num_threads", 1)) for i in threadpool_info()) or 1
     except Exception:
+        if os.environ.get("OMP_NUM_THREADS") == "1":
+            return 1
         return os.cpu_count() or 1
 
 
-def cpu_baseline(B: int, budget_s: float = 20.0, linears=None):
-    """The oracle's wl_matmul (float64 numpy, as it stands) on the host cores, over the
-    linears of decoder layer 0 in order until the time budget is used (at least one linear)."""
+def oracle_sample(B: int, count: int = SAMPLE_LINEARS):
+    """The oracle's inputs for the bounded sample: layer 0's first `count` linears at batch B."""
+    shapes = layer_shapes(1)[:max(1, count)]
+    return [(rows, cols, name, _oracle_layer(rows, cols, synth.weight_seed("stack", L, pi), B))
+            for (L, pi, name, rows, cols) in shapes]
+
+
+def time_oracle(prepared, budget_s: float):
+    """Passes of the oracle's wl_matmul (float64 numpy, as it stands) over the sample until the
+    time budget is used (at least one pass): GB/s of the algorithmic bytes."""
     import oracle as O
-    shapes = layer_shapes(1) if linears is None else linears
-    done_bytes, spent, names = 0, 0.0, []
-    for (L, pi, name, rows, cols) in shapes:
-        codes, scales, x = _oracle_layer(rows, cols, synth.weight_seed("stack", L, pi), B)
+    B = prepared[0][3][2].shape[0]
+    nbytes = sum(layer_bytes(r, c, B) for r, c, _, _ in prepared)
+    passes, spent = 0, 0.0
+    while passes == 0 or spent < budget_s:
         t0 = time.perf_counter()
-        O.wl_matmul(x, codes, scales, rows)
+        for rows, cols, _, (codes, scales, x) in prepared:
+            O.wl_matmul(x, codes, scales, rows)
         spent += time.perf_counter() - t0
-        done_bytes += layer_bytes(rows, cols, B)
-        names.append(f"{L}.{name}")
-        if spent >= budget_s:
-            break
-    return {"value": round(done_bytes / spent / 1e9, 4), "unit": "GB/s", "cores": _threads(),
-            "kind": "oracle",
-            "sample": f"oracle wl_matmul over linears {','.join(names)} of the stack, batch {B} "
-                      f"({spent:.1f} s; setup (oracle convert+quantize) untimed)"}
+        passes += 1
+    return nbytes * passes / spent / 1e9, passes, spent
+
+
+def cpu_baseline(B: int, budget_s: float = 10.0, count: int = SAMPLE_LINEARS):
+    """The oracle on the host cores: BLAS with its default threads (all cores) in this process,
+    and one thread in a child process started with the thread-count variables set to 1."""
+    prepared = oracle_sample(B, count)
+    gbs, passes, spent = time_oracle(prepared, budget_s)
+    names = ",".join(f"0.{nm}" for _, _, nm, _ in prepared)
+    res = {"value": round(gbs, 5), "unit": "GB/s", "cores": _threads(), "kind": "oracle",
+           "sample": f"oracle wl_matmul over linears {names} of the stack, batch {B}, "
+                     f"{passes} passes ({spent:.1f} s); setup (oracle convert+quantize) untimed"}
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    try:
+        out = subprocess.run([sys.executable, os.path.abspath(__file__), "--oracle-sample-only",
+                              "--batch", str(B), "--cpu-budget", str(budget_s),
+                              "--ref-linears", str(count)],
+                             env=env, capture_output=True, text=True, timeout=600)
+        one = json.loads(out.stdout.strip().splitlines()[-1])
+        res["one_thread"] = {"value": one["value"], "unit": "GB/s", "cores": 1,
+                             "sample": one["sample"]}
+    except Exception as e:   # noqa: BLE001
+        res["one_thread"] = {"unavailable": f"{type(e).__name__}"}
+    return res
 
 
 def run_reference(args, world, rank):
     if rank != 0:
         return None
-    import oracle  # noqa: F401
-    shapes = layer_shapes(1)
-    per_step = shapes[: max(1, args.ref_linears)]
-    prepared = [(rows, cols, _oracle_layer(rows, cols, synth.weight_seed("stack", L, pi), args.batch))
-                for (L, pi, name, rows, cols) in per_step]
+    prepared = oracle_sample(args.batch, args.ref_linears)
     import oracle as O
 
     def step():
-        for rows, cols, (codes, scales, x) in prepared:
+        for rows, cols, _, (codes, scales, x) in prepared:
             O.wl_matmul(x, codes, scales, rows)
 
     for _ in range(args.warmup):
@@ -504,21 +734,21 @@ def run_reference(args, world, rank):
     for _ in range(args.steps):
         step()
     sec = time.perf_counter() - t0
-    step_bytes = sum(layer_bytes(r, c, args.batch) for r, c, _ in prepared)
+    step_bytes = sum(layer_bytes(r, c, args.batch) for r, c, _, _ in prepared)
     value = step_bytes * args.steps / sec / 1e9
-    names = ",".join(f"0.{n}" for (_, _, n, _, _) in per_step)
+    names = ",".join(f"0.{nm}" for _, _, nm, _ in prepared)
     return {
-        "impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": "GB/s",
+        "impl": "reference", "metric": METRIC, "value": round(value, 5), "unit": "GB/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(sec / args.steps * 1e3, 3), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic (same seeds as the GPU arm)",
         "config": {"workload": WORKLOAD, "layers": args.layers, "T": T_STAGES,
                    "batch": args.batch, "x_dtype": "bf16",
-                   "sample_per_step": f"linears {names} (bounded sample of the stack)"},
-        "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
+                   "sample_per_step": f"linears {names} (the bounded sample cpu_baseline times)"},
+        "e2e": {"value": round(value, 5), "unit": "GB/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
-        "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": _threads(),
+        "cpu_baseline": {"value": round(value, 5), "unit": "GB/s", "cores": _threads(),
                          "kind": "oracle", "sample": f"linears {names} per step"},
     }
 
@@ -533,14 +763,29 @@ def main():
     ap.add_argument("--layers", type=int, default=32)
     ap.add_argument("--no-graph", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--cpu-budget", type=float, default=15.0)
-    ap.add_argument("--ref-linears", type=int, default=2)
+    ap.add_argument("--cpu-budget", type=float, default=8.0)
+    ap.add_argument("--ref-linears", type=int, default=SAMPLE_LINEARS,
+                    help="linears of layer 0 in the oracle sample (cpu_baseline, reference arm)")
     ap.add_argument("--no-prefill", action="store_true")
+    ap.add_argument("--no-sweep", action="store_true")
+    ap.add_argument("--no-chain", action="store_true")
+    ap.add_argument("--no-quantize", action="store_true")
+    ap.add_argument("--no-lut", action="store_true")
     ap.add_argument("--ungrouped", action="store_true")
     ap.add_argument("--prefill-steps", type=int, default=10)
-    ap.add_argument("--decode-path", type=int, default=0, choices=[0, 1, 4],
-                    help="decode kernel: 0 automatic, 1 warp-MMA, 4 persistent tcgen05")
+    ap.add_argument("--oracle-sample-only", action="store_true", help=argparse.SUPPRESS)
+    ap.add_argument("--decode-path", type=int, default=0, choices=[0, 1, 4, 5],
+                    help="decode kernel: 0 automatic, 1 warp-MMA, 4 persistent tcgen05, "
+                         "5 chained kernel per call")
     args = ap.parse_args()
+    if args.oracle_sample_only:
+        prepared = oracle_sample(args.batch, args.ref_linears)
+        gbs, passes, spent = time_oracle(prepared, args.cpu_budget)
+        names = ",".join(f"0.{nm}" for _, _, nm, _ in prepared)
+        print(json.dumps({"value": round(gbs, 5),
+                          "sample": f"linears {names}, batch {args.batch}, {passes} passes "
+                                    f"({spent:.1f} s), one thread"}))
+        return
     world, rank, local = dist_setup()
     if args.impl == "reference":
         line = run_reference(args, world, rank)

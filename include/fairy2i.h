@@ -162,10 +162,12 @@ fairy2i_status fairy2i_wl_matmul(const void* x, fairy2i_dtype xdt, int64_t B,
                                  int64_t ldy, void* stream);
 
 /* Same as fairy2i_wl_matmul with the kernel chosen by `path`:
- *   0 = automatic: B <= 2 bf16 tokens and T <= 4 -> a decode kernel: the persistent tcgen05 one
- *       (4) when the call's 16-row tiles outnumber the SMs, else the warp-MMA one (1); B > 2 ->
+ *   0 = automatic: B <= 2 -> one token at a time through a decode kernel that meets the
+ *       per-element bound for any x: the persistent tcgen05 kernel's one-token form (4) for bf16
+ *       x, the chained kernel (5) for float32 x (both T <= 4, in_features <= 24576); B > 2 ->
  *       the tcgen05 prefill GEMM where it applies (see 3); otherwise the general CUDA-core kernel;
- *   1 = the decode kernel where it applies, otherwise the general kernel;
+ *   1 = the warp-MMA decode kernel (x as two e4m3 limbs, B <= 2) where it applies, otherwise
+ *       the general kernel;
  *   2 = retired (an earlier tcgen05 decode kernel); returns FAIRY2I_ERR_INVALID_ARG;
  *   3 = the tcgen05 prefill GEMM (codes expanded into bf16 +-1 tiles in tensor memory, x by TMA,
  *       64 tokens per tile); it takes bf16 x with 16-byte aligned rows, ldx % 8 == 0,
@@ -214,14 +216,13 @@ fairy2i_status fairy2i_codes_adjoint(const uint32_t* codes, int64_t n, int64_t m
  * or the gate and up projections of a decoder layer: for g < count,
  *   y[g] = fairy2i_wl_matmul(x, xdt, B, in_features, ldx, codes[g], scales[g], out_features, T)
  * with codes[g], scales[g], y[g] device pointers passed in host arrays of `count` entries
- * (1 <= count <= FAIRY2I_MAX_GROUP). Where a decode kernel applies (B <= 2 bf16 tokens,
- * T <= 4) the whole group is one launch, of the persistent tcgen05 kernel when the group's 16-row
- * tiles outnumber the SMs, else of the warp-MMA kernel; otherwise the members run one after the
- * other on the automatic path. Requirements and errors are those of fairy2i_wl_matmul for every
- * member (checked before anything is enqueued); FAIRY2I_ERR_INVALID_ARG for a count out of range
- * or a null array. Results agree with the separate calls within the float32-accumulation
- * tolerance (the kernel may differ: a group has more tiles than each member); on the warp-MMA
- * kernel they are bit-identical.
+ * (1 <= count <= FAIRY2I_MAX_GROUP). Where the automatic decode path applies (B <= 2, T <= 4,
+ * in_features <= 24576) the whole group is one launch per token (the persistent tcgen05 kernel's
+ * one-token form for bf16 x, the chained kernel for float32 x); otherwise the members run one
+ * after the other on the automatic path. Requirements and errors are those of fairy2i_wl_matmul
+ * for every member (checked before anything is enqueued); FAIRY2I_ERR_INVALID_ARG for a count
+ * out of range or a null array. Results agree with the separate calls within the
+ * float32-accumulation tolerance (a group splits its work over the SMs differently).
  * ------------------------------------------------------------------------------------------ */
 #define FAIRY2I_MAX_GROUP 4
 fairy2i_status fairy2i_wl_matmul_group(const void* x, fairy2i_dtype xdt, int64_t B,
@@ -231,7 +232,7 @@ fairy2i_status fairy2i_wl_matmul_group(const void* x, fairy2i_dtype xdt, int64_t
                                        void* stream);
 
 /* fairy2i_wl_matmul_group with the decode kernel chosen by `path`: 0 = automatic (as above),
- * 1 = the warp-MMA decode kernel where it applies (else the automatic path per member),
+ * 1 = the warp-MMA decode kernel where it applies (else path 1 per member),
  * 4 = the persistent tcgen05 decode kernel, one launch for the group (B <= 2 bf16 tokens, T <= 4,
  * in_features <= 24576; FAIRY2I_ERR_INVALID_ARG for anything else), 5 = the chained decode kernel
  * on this one group (B = 1, T <= 4, in_features <= 24576; FAIRY2I_ERR_INVALID_ARG otherwise).

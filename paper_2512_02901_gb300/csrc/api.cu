@@ -82,21 +82,50 @@ unsigned int* device_status_word() {
 
 static bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
-// Automatic choice between the two decode kernels (B <= 2 bf16 tokens): the warp-MMA kernel
-// gives each 16-row tile its own CTA, so once the tiles of the call outnumber the SMs it runs in
-// several waves and the persistent tcgen05 kernel (one wave, every CTA looping over row blocks)
-// is faster; with at most one wave the warp-MMA kernel's shorter launch wins.
-static bool prefer_stream(int64_t n, int count) {
-  static std::atomic<int> sms[64];   // per device, 0 = not read yet
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
-  int v = sms[dev].load(std::memory_order_relaxed);
-  if (!v) {
-    if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || v < 1)
-      return false;
-    sms[dev].store(v, std::memory_order_relaxed);
+// The automatic decode path (B <= 2 tokens): one token at a time through a kernel that holds
+// every x entry to the per-element bound for any x, i.e. to 2^-26 (persistent tcgen05 kernel,
+// one-token form, bf16 x) or 2^-28 (chained kernel, float32 x) of the largest |x| in the K slice
+// one CTA handles (at most 3072 and 12288 values). *handled = false (nothing launched) where
+// neither kernel takes the shape.
+static fairy2i_status auto_decode(const void* x, fairy2i_dtype xdt, int64_t B, int64_t in_features,
+                                  int64_t ldx, int count, const uint32_t* const* codes,
+                                  const float* const* scales, int64_t n, int64_t m,
+                                  int64_t out_features, int64_t wpr, int T, float* const* y,
+                                  int64_t ldy, cudaStream_t s, bool* handled) {
+  *handled = false;
+  const int64_t esz = xdt == FAIRY2I_BF16 ? 2 : 4;
+  if (xdt == FAIRY2I_F32) {   // chained kernel: T <= 4, in_features <= 24576, x 16-byte aligned
+    if (T > 4 || in_features > 24576 || (B > 1 && (ldx * esz) % 16 != 0)) return FAIRY2I_OK;
   }
-  return (int64_t)count * ((n + 15) / 16) > v;
+  for (int64_t b = 0; b < B; ++b) {
+    const void* xb = static_cast<const char*>(x) + b * ldx * esz;
+    float* yb[FAIRY2I_MAX_GROUP];
+    for (int g = 0; g < count; ++g) yb[g] = y[g] + b * ldy;
+    if (xdt == FAIRY2I_BF16) {
+      bool h = false;
+      const fairy2i_status st = launch_wl_stream_group(xb, xdt, 1, in_features, ldx, count, codes,
+                                                       scales, n, m, out_features, wpr, T, yb,
+                                                       ldy, s, &h);
+      if (st != FAIRY2I_OK) return st;
+      if (!h) return FAIRY2I_OK;   // the same shape for every token: only b = 0 gets here
+    } else {
+      fairy2i_chain_call c = {};
+      c.x = xb;
+      c.xdt = xdt;
+      c.count = count;
+      c.in_features = in_features;
+      c.out_features = out_features;
+      for (int g = 0; g < count; ++g) {
+        c.codes[g] = codes[g];
+        c.scales[g] = scales[g];
+        c.y[g] = yb[g];
+      }
+      const fairy2i_status st = fairy2i_wl_matmul_chain(&c, 1, T, 0, nullptr, 0, s);
+      if (st != FAIRY2I_OK) return st;
+    }
+  }
+  *handled = true;
+  return FAIRY2I_OK;
 }
 
 }  // namespace fairy2i
@@ -200,14 +229,16 @@ fairy2i_status fairy2i_wl_matmul_path(const void* x, fairy2i_dtype xdt, int64_t 
     c.y[0] = y;
     return fairy2i_wl_matmul_chain(&c, 1, T, 0, nullptr, 0, stream);
   }
-  if (path == 0 && B <= 2 && xdt == FAIRY2I_BF16 && prefer_stream(n, 1)) {
-    st = launch_wl_stream_group(x, xdt, B, in_features, ldx, 1, &codes, &scales, n, m,
-                                out_features, wpr, T, &y, ldy, s, &handled);
+  if (path == 0 && B <= 2) {
+    st = auto_decode(x, xdt, B, in_features, ldx, 1, &codes, &scales, n, m, out_features, wpr, T,
+                     &y, ldy, s, &handled);
     if (handled || st != FAIRY2I_OK) return st;
   }
-  st = launch_wl_decode(x, xdt, B, in_features, ldx, codes, scales, n, m,
-                                       out_features, wpr, T, y, ldy, s, &handled);
-  if (handled || st != FAIRY2I_OK) return st;
+  if (path == 1) {   // warp-MMA decode kernel (explicit): e4m3 limbs of x
+    st = launch_wl_decode(x, xdt, B, in_features, ldx, codes, scales, n, m, out_features, wpr, T,
+                          y, ldy, s, &handled);
+    if (handled || st != FAIRY2I_OK) return st;
+  }
   return launch_wl_simple(x, xdt, B, in_features, ldx, codes, scales, n, m, out_features, wpr, T,
                           y, ldy, s);
 }
@@ -259,24 +290,28 @@ fairy2i_status fairy2i_wl_matmul_group_path(const void* x, fairy2i_dtype xdt, in
   const int64_t wpr = fairy2i_codes_words_per_row(m);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   bool handled = false;
-  if (B <= 2 && (path == 4 || (path == 0 && xdt == FAIRY2I_BF16 && prefer_stream(n, count)))) {
-    // one launch of the persistent tcgen05 decode kernel
+  if (B <= 2 && path == 0) {   // per token, one launch for the whole group
+    const fairy2i_status st = auto_decode(x, xdt, B, in_features, ldx, count, codes, scales, n, m,
+                                          out_features, wpr, T, y, ldy, s, &handled);
+    if (handled || st != FAIRY2I_OK) return st;
+  }
+  if (B <= 2 && path == 4) {   // one launch of the persistent tcgen05 decode kernel
     const fairy2i_status st = launch_wl_stream_group(x, xdt, B, in_features, ldx, count, codes,
                                                      scales, n, m, out_features, wpr, T, y, ldy,
                                                      s, &handled);
     if (handled || st != FAIRY2I_OK) return st;
-    if (path == 4) return FAIRY2I_ERR_INVALID_ARG;
+    return FAIRY2I_ERR_INVALID_ARG;
   }
-  if (B <= 2) {   // one launch of the warp-MMA decode kernel for the whole group
+  if (B <= 2 && path == 1) {   // one launch of the warp-MMA decode kernel for the whole group
     const fairy2i_status st = launch_wl_decode_group(x, xdt, B, in_features, ldx, count, codes,
                                                      scales, n, m, out_features, wpr, T, y, ldy,
                                                      s, &handled);
     if (handled || st != FAIRY2I_OK) return st;
   }
-  for (int g = 0; g < count; ++g) {   // elsewhere: the automatic path per member
+  for (int g = 0; g < count; ++g) {   // elsewhere: per member
     const fairy2i_status st = fairy2i_wl_matmul_path(x, xdt, B, in_features, ldx, codes[g],
-                                                     scales[g], out_features, T, y[g], ldy, 0,
-                                                     stream);
+                                                     scales[g], out_features, T, y[g], ldy,
+                                                     path == 1 ? 1 : 0, stream);
     if (st != FAIRY2I_OK) return st;
   }
   return FAIRY2I_OK;

@@ -164,27 +164,58 @@ def test_stream_rejects_outside_its_domain(F):
     assert F.get_status() == 0
 
 
-def test_automatic_path_routes_by_tile_count(F):
-    """The automatic decode path takes the persistent kernel when a call's 16-row tiles outnumber
-    the SMs (here the grouped q/k/v shape: 3 x 128 tiles) and the warp-MMA kernel otherwise (one
-    4096 -> 4096 linear: 128 tiles): bit for bit the results of the explicit paths, both kernels
-    being deterministic."""
-    sms = torch.cuda.get_device_properties(0).multi_processor_count
+def test_automatic_decode_runs_the_one_token_kernel_per_token(F):
+    """The automatic decode path (B <= 2, bf16 x) runs the persistent kernel's one-token form
+    token by token, one launch per token for a whole group: bit for bit the results of explicit
+    one-token path-4 calls (the kernel is deterministic and a token's result does not depend on
+    the other token)."""
     out_f, in_f, T = 4096, 4096, 2
     n, m = O.complex_dims(out_f, in_f)
-    assert 3 * ((n + 15) // 16) > sms >= (n + 15) // 16
     layers = [_random_quantized(n, m, T, seed=81 + g) for g in range(3)]
     cds = [_upload(c) for c, _ in layers]
     scs = [torch.from_numpy(s).to(DEV) for _, s in layers]
-    x = synth.outlier_activations(1, in_f, seed=83).to(DEV)
+    x = synth.outlier_activations(2, in_f, seed=83).to(DEV)
     auto_group = F.wl_matmul_group(x, cds, scs, out_f)
-    stream_group = F.wl_matmul_group(x, cds, scs, out_f, path=PATH)
     auto_single = F.wl_matmul(x, cds[0], scs[0], out_f)
-    warp_single = F.wl_matmul(x, cds[0], scs[0], out_f, path=1)
+    for b in range(2):
+        xb = x[b:b + 1].contiguous()
+        per_token = F.wl_matmul_group(xb, cds, scs, out_f, path=PATH)
+        for a, p in zip(auto_group, per_token):
+            assert torch.equal(a[b:b + 1], p)
+        assert torch.equal(auto_single[b:b + 1], F.wl_matmul(xb, cds[0], scs[0], out_f, path=PATH))
     assert F.get_status() == 0
-    for a, b in zip(auto_group, stream_group):
-        assert torch.equal(a, b)
-    assert torch.equal(auto_single, warp_single)
+
+
+@pytest.mark.parametrize("out_f,in_f,B,dtype", [
+    (4096, 11008, 1, torch.bfloat16),    # the 7B down projection
+    (11008, 4096, 1, torch.bfloat16),    # the 7B gate / up projections
+    (4096, 4096, 2, torch.bfloat16),     # two tokens
+    (4096, 11008, 1, torch.float32),     # float32 x: the chained kernel
+    (4096, 4096, 2, torch.float32),
+])
+def test_automatic_decode_element_bound_for_extreme_x(F, out_f, in_f, B, dtype):
+    """Every output of the automatic decode path stays within the per-element bound
+    1e-4 |x~|_1 sum_t s_t whatever x is. Worst case for the fixed-point forms: x = (1, tiny,
+    tiny, ...) with the tiny entries just under half a unit of the grid (2^-26 of the slice
+    maximum for bf16 x, 2^-28 for float32 x; the second token scaled by 2^-10 with its own tiny
+    entries), every code +1 so that the rounding errors add up in every row."""
+    T = 2
+    n, m = O.complex_dims(out_f, in_f)
+    codes = np.zeros((T, 2, n, m), dtype=np.uint8)
+    scales = np.full((T, 2, 2), 0.02, dtype=np.float32)
+    unit = 2.0 ** -26 if dtype == torch.bfloat16 else 2.0 ** -28
+    x = torch.full((B, in_f), 0.99609375 * unit, dtype=torch.float32)
+    x[0, 0] = 1.0
+    if B > 1:
+        x[1] = 2.0 ** -10 * 0.99609375 * unit * 4
+        x[1, 7] = -(2.0 ** -10)
+    x = x.to(dtype)
+    y = F.wl_matmul(x.to(DEV), _upload(codes), torch.from_numpy(scales).to(DEV), out_f)
+    assert F.get_status() == 0
+    xo = x.float().numpy().astype(np.float64)
+    err = np.asarray(y.cpu().numpy(), np.float64) - O.wl_matmul(xo, codes, scales, out_f)
+    bound = 1e-4 * O.tolerance_bound(xo, scales)[:, None]
+    assert np.max(np.abs(err) - bound) <= 0, f"element error {np.max(np.abs(err) / bound):.3f} of the bound"
 
 
 @pytest.mark.parametrize("tiny", [0.99609375 * 2.0**-24, 0.99609375 * 2.0**-26])
