@@ -117,7 +117,7 @@ fairy2i_status fairy2i_quantize(const float* U, const float* W, int64_t n, int64
  * GPU that loads the library holds until the process exits. The call allocates nothing and
  * calls no allocating routine.
  *  - Sizes: fairy2i_quantize_workspace_bytes(n, m, T) must not exceed the array, i.e.
- *    n*m <= 16,646,656 complex weights per matrix (a 4096 -> 11008 layer, 5504 x 2048, fits);
+ *    n*m <= 16,703,232 complex weights per matrix (a 4096 -> 11008 layer, 5504 x 2048, fits);
  *    larger sizes return FAIRY2I_ERR_WORKSPACE and enqueue nothing.
  *  - The first call on a device looks up the array's device address (cudaGetSymbolAddress,
  *    with that device current); make that first call before any stream capture on the device.
@@ -128,7 +128,8 @@ fairy2i_status fairy2i_quantize(const float* U, const float* W, int64_t n, int64
  *    calls commit nothing).
  *  - All calls share the one array, on every stream: calls whose kernels overlap on the GPU
  *    (different streams without ordering between them) race and give wrong results. Calls
- *    ordered on one stream are safe; each call writes every scratch entry before reading it.
+ *    ordered on one stream are safe; each call writes every scratch entry before reading it
+ *    (its completion counters are cleared by the call itself).
  * ------------------------------------------------------------------------------------------ */
 #define FAIRY2I_NOALLOC_SCRATCH_BYTES (4u << 20)
 fairy2i_status fairy2i_quantize_noalloc(const float* U, const float* W, int64_t n, int64_t m,

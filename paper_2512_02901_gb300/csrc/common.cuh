@@ -28,10 +28,13 @@ __device__ __forceinline__ unsigned project_code(float a, float b) {
 // Residual update of Sec. 3.3: r -= s_re b_re + i s_im b_im, one IEEE add per element.
 __device__ __forceinline__ void residual_update(float& a, float& b, unsigned c, float s_re,
                                                 float s_im) {
-  if (c == 0u) a = __fsub_rn(a, s_re);
-  else if (c == 2u) a = __fadd_rn(a, s_re);
-  else if (c == 1u) b = __fsub_rn(b, s_im);
-  else b = __fadd_rn(b, s_im);
+  // c even: a -= (1 - c) s_re; c odd: b -= (2 - c) s_im (selects, no branches)
+  const bool odd = (c & 1u) != 0u;
+  const float sg = (c & 2u) ? -1.f : 1.f;
+  const float d = sg * (odd ? s_im : s_re);   // exact: a sign flip
+  const float nv = __fsub_rn(odd ? b : a, d);
+  a = odd ? a : nv;
+  b = odd ? nv : b;
 }
 
 // Packed bit pair of a code: (Re+Im < 0, Re-Im < 0) of the codeword.

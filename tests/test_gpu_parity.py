@@ -135,6 +135,30 @@ def test_quantize_nonfinite_latches_status(F):
     assert F.get_status() == 0          # read clears
 
 
+def test_quantize_wide_range_values(F):
+    """Values spread over ~60 binades (and some subnormal): most 256-element groups take the
+    float64 tree instead of the exact integer sum, some groups mix both cases across the two
+    sums; codes and scales still bit-exact."""
+    g = np.random.default_rng(21)
+    n, m = 96, 1000
+    def wide():
+        mag = g.standard_normal((n, m)) * np.exp2(g.integers(-40, 21, (n, m)))
+        mag[g.random((n, m)) < 0.01] = 3e-42            # float32 subnormals
+        return mag
+    U = (wide() + 1j * 0.02 * g.standard_normal((n, m))).astype(np.complex64)
+    W = (0.02 * g.standard_normal((n, m)) + 1j * wide()).astype(np.complex64)
+    _assert_quant_equal(*_quantize_both(F, U, W, 3))
+
+
+def test_quantize_three_reduction_levels(F):
+    """n m > 2^24: more than 256 level-1 groups, so the scales take a third tree level."""
+    g = np.random.default_rng(23)
+    n, m = 4100, 4100
+    U = (0.02 * g.standard_normal((n, m)) + 0.02j * g.standard_normal((n, m))).astype(np.complex64)
+    W = (0.02 * g.standard_normal((n, m)) - 0.01j * g.standard_normal((n, m))).astype(np.complex64)
+    _assert_quant_equal(*_quantize_both(F, U, W, 1))
+
+
 @pytest.mark.parametrize("rows,cols,T,seed", [
     (4096, 4096, 2, synth.weight_seed("attn")),             # attention projection, decode
     (11008, 4096, 2, synth.weight_seed("mlp", 0)),          # up / gate

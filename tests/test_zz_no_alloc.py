@@ -52,6 +52,6 @@ def test_noalloc_matches_workspace_quantizer_twice(F):
 def test_noalloc_rejects_sizes_beyond_scratch(F):
     P = ctypes.c_void_p(1 << 20)
     lib = F.load()
-    # 4096 x 4065 = 16,650,240 complex weights: just beyond the 4 MiB scratch
-    assert lib.fairy2i_quantize_noalloc(P, P, 4096, 4065, 4065, 2, P, P, None) == 5
+    # 4096 x 4078 = 16,703,488 complex weights: just beyond the 4 MiB scratch (16,703,232 fit)
+    assert lib.fairy2i_quantize_noalloc(P, P, 4096, 4078, 4078, 2, P, P, None) == 5
     assert lib.fairy2i_quantize_noalloc(P, P, 8, 8, 8, 0, P, P, None) == 1
