@@ -316,8 +316,10 @@ def run_ours(args, world, rank, local):
     calls, x_all, y_all = make_calls(linears, B, dev, groups)
     step_bytes = sum(call_bytes(c, B) for c in calls)
     nlinears = sum(len(c["members"]) for c in calls)
-    # a grouped call is one launch where the decode kernel takes it (B <= 2), else one per member
-    launches_per_step = len(calls) if B <= 2 else nlinears
+    # a grouped call is one launch per token (B = 1) or per 4 tokens (2 <= B <= 8) where a decode
+    # kernel takes it, else one per member
+    launches_per_step = (len(calls) if B == 1 else len(calls) * ((B + 3) // 4) if B <= 8
+                         else nlinears)
 
     def step():
         for c in calls:
@@ -387,7 +389,8 @@ def run_ours(args, world, rank, local):
     achieved = step_bytes / (ms_step * 1e-3) / 1e9
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
     traffic = decode_traffic(calls, args.decode_path, B, sms)
-    kernels = sorted({decode_kernel(c, args.decode_path, sms) for c in calls}) if B <= 2 else []
+    kernels = (sorted({decode_kernel(c, args.decode_path, sms) for c in calls}) if B == 1 else
+               ["chain"] if B <= 8 and args.decode_path in (0, 5) else [])
     kname = ("wl_matmul decode (all launches of the step: "
              + " + ".join({"fp8": "warp-MMA", "stream": "persistent tcgen05",
                            "chain": "chained tcgen05"}[k] for k in kernels)
@@ -495,7 +498,9 @@ def run_batches(F, linears, dev, args):
             rec["us_per_linear"] = round(ms * 1e3 / nlin, 2)
         if name.startswith("mlp"):
             rec["us_per_layer"] = round(ms * 1e3 / len(linears), 2)
-        rec["path"] = "decode kernels" if B <= 2 else "tcgen05 GEMM (64-token tiles)"
+        rec["path"] = ("persistent tcgen05, one-token form" if B == 1 else
+                       "chained tcgen05, up to 4 tokens per launch" if B <= 8 else
+                       "tcgen05 GEMM (64-token tiles)")
         out.append(rec)
         del calls, x_all, y_all
     torch.cuda.empty_cache()

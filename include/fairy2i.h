@@ -147,13 +147,14 @@ fairy2i_status fairy2i_quantize_noalloc(const float* U, const float* W, int64_t 
  *   codes, scales  as written by fairy2i_quantize for (n, m, T), n = ceil(out_features/2).
  *   y     float32 [B][ldy], overwritten: y[0:n] = Re y, y[n:out_features] = Im y.
  *   Accuracy: every kernel accumulates in fp32. The general (fp32 x) and prefill kernels use x
- *   exactly; the decode kernels (bf16 x, B <= 2) hold each x entry in fixed point relative to
- *   the largest |x| of the part of the K range one warp or CTA handles: the one-token
- *   persistent kernel to half a unit of 2^-25 of it, the e4m3 kernels (warp-MMA, two-token
- *   persistent) exactly down to ~2^-13 of it and to ~2^-22 below. Each output is then
- *   within 1e-4 |x~|_1 sum_t max(s_re, s_im) (U and W terms) of the float64 value for any x on
- *   the fp32, prefill and one-token persistent kernels, and on the e4m3 kernels unless hundreds
- *   of entries of one part lie in (0, ~2^-13) of its maximum. Non-finite x: y unspecified.
+ *   exactly; the decode kernels hold each x entry in fixed point relative to the largest |x| of
+ *   its token in the part of the K range one warp or CTA handles: the one-token persistent
+ *   kernel to half a unit of 2^-25 of it, the chained kernel to half a unit of 2^-27, the e4m3
+ *   kernels (warp-MMA, two-token persistent: explicit paths only) exactly down to ~2^-13 of it
+ *   and to ~2^-22 below. Each output is then within 1e-4 |x~|_1 sum_t max(s_re, s_im) (U and W
+ *   terms) of the float64 value for any x on every kernel the automatic path runs, and on the
+ *   e4m3 kernels unless hundreds of entries of one part lie in (0, ~2^-13) of its maximum.
+ *   Non-finite x: y unspecified.
  *   Requirements: B >= 0 (B = 0 is a no-op), in_features, out_features >= 1, 1 <= T <= 8,
  *   ldx >= in_features, ldy >= out_features, codes and x 16-byte aligned, y 4-byte aligned.
  * ------------------------------------------------------------------------------------------ */
@@ -163,10 +164,11 @@ fairy2i_status fairy2i_wl_matmul(const void* x, fairy2i_dtype xdt, int64_t B,
                                  int64_t ldy, void* stream);
 
 /* Same as fairy2i_wl_matmul with the kernel chosen by `path`:
- *   0 = automatic: B <= 2 -> one token at a time through a decode kernel that meets the
- *       per-element bound for any x: the persistent tcgen05 kernel's one-token form (4) for bf16
- *       x, the chained kernel (5) for float32 x (both T <= 4, in_features <= 24576); B > 2 ->
- *       the tcgen05 prefill GEMM where it applies (see 3); otherwise the general CUDA-core kernel;
+ *   0 = automatic, every decode choice meeting the per-element bound for any x: B = 1 -> the
+ *       persistent tcgen05 kernel's one-token form (4) for bf16 x, the chained kernel (5) for
+ *       float32 x; 2 <= B <= 8 -> the chained kernel, up to 4 tokens per launch (skinny batch);
+ *       (decode kernels: T <= 4, in_features <= 24576); B > 8 -> the tcgen05 prefill GEMM where
+ *       it applies (see 3); otherwise the general CUDA-core kernel;
  *   1 = the warp-MMA decode kernel (x as two e4m3 limbs, B <= 2) where it applies, otherwise
  *       the general kernel;
  *   2 = retired (an earlier tcgen05 decode kernel); returns FAIRY2I_ERR_INVALID_ARG;
@@ -181,8 +183,9 @@ fairy2i_status fairy2i_wl_matmul(const void* x, fairy2i_dtype xdt, int64_t B,
  *       which keeps every output within the per-element bound for any x; two tokens: e4m3
  *       operands, x as two e4m3 limbs); it takes B <= 2 bf16 tokens, T <= 4 and
  *       in_features <= 24576 and returns FAIRY2I_ERR_INVALID_ARG for anything else;
- *   5 = the chained decode kernel (fairy2i_wl_matmul_chain) on this one call; it takes B = 1
- *       token (float32 or bf16), T <= 4 and in_features <= 24576 and returns
+ *   5 = the chained decode kernel (fairy2i_wl_matmul_chain) on this one call, up to 4 tokens
+ *       per launch (the decoded signs feed the MMAs of every token of the launch); it takes any
+ *       B (float32 or bf16 x), T <= 4 and in_features <= 24576 and returns
  *       FAIRY2I_ERR_INVALID_ARG for anything else.
  * The decode kernels (paths 1, 4) read the codes and scales before waiting for the previous
  * kernel in the stream (programmatic dependent launch): the codes must not be written by the
@@ -217,10 +220,10 @@ fairy2i_status fairy2i_codes_adjoint(const uint32_t* codes, int64_t n, int64_t m
  * or the gate and up projections of a decoder layer: for g < count,
  *   y[g] = fairy2i_wl_matmul(x, xdt, B, in_features, ldx, codes[g], scales[g], out_features, T)
  * with codes[g], scales[g], y[g] device pointers passed in host arrays of `count` entries
- * (1 <= count <= FAIRY2I_MAX_GROUP). Where the automatic decode path applies (B <= 2, T <= 4,
- * in_features <= 24576) the whole group is one launch per token (the persistent tcgen05 kernel's
- * one-token form for bf16 x, the chained kernel for float32 x); otherwise the members run one
- * after the other on the automatic path. Requirements and errors are those of fairy2i_wl_matmul
+ * (1 <= count <= FAIRY2I_MAX_GROUP). Where the automatic decode path applies (B <= 8, T <= 4,
+ * in_features <= 24576) the whole group is one launch per token (B = 1: the persistent tcgen05
+ * kernel's one-token form for bf16 x, the chained kernel for float32 x) or per 4 tokens (the
+ * chained kernel); otherwise the members run one after the other on the automatic path. Requirements and errors are those of fairy2i_wl_matmul
  * for every member (checked before anything is enqueued); FAIRY2I_ERR_INVALID_ARG for a count
  * out of range or a null array. Results agree with the separate calls within the
  * float32-accumulation tolerance (a group splits its work over the SMs differently).
@@ -236,7 +239,8 @@ fairy2i_status fairy2i_wl_matmul_group(const void* x, fairy2i_dtype xdt, int64_t
  * 1 = the warp-MMA decode kernel where it applies (else path 1 per member),
  * 4 = the persistent tcgen05 decode kernel, one launch for the group (B <= 2 bf16 tokens, T <= 4,
  * in_features <= 24576; FAIRY2I_ERR_INVALID_ARG for anything else), 5 = the chained decode kernel
- * on this one group (B = 1, T <= 4, in_features <= 24576; FAIRY2I_ERR_INVALID_ARG otherwise).
+ * on this one group (any B, up to 4 tokens per launch, T <= 4, in_features <= 24576;
+ * FAIRY2I_ERR_INVALID_ARG otherwise).
  * Any other path returns
  * FAIRY2I_ERR_INVALID_ARG. Results agree with the separate calls within the float32-accumulation
  * tolerance (bit-identical for path 1). */

@@ -34,7 +34,8 @@ fairy2i_status launch_wl_stream_group(const void* x, fairy2i_dtype xdt, int64_t 
                                       bool* handled);
 fairy2i_status launch_selftest_wait(uint32_t limit_us, cudaStream_t stream);
 fairy2i_status launch_wl_chain(const fairy2i_chain_call* calls, int ncalls, int T,
-                               int cluster_size, unsigned int* done, cudaStream_t stream);
+                               int cluster_size, unsigned int* done, cudaStream_t stream,
+                               int nb = 1, int64_t ldx = 0, int64_t ldy = 0);
 int chain_max_calls();
 size_t ste_grad_workspace_bytes(int64_t B, int64_t in_features, int64_t out_features);
 fairy2i_status launch_ste_grad(const void* x, int64_t ldx, const void* g, int64_t ldg, int64_t B,
@@ -82,6 +83,10 @@ unsigned int* device_status_word() {
 
 static bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
+// Largest batch the automatic path sends to the chained kernel (skinny-batch decode); larger
+// batches take the tcgen05 prefill GEMM.
+constexpr int64_t kSkinnyMaxTokens = 8;
+
 // The automatic decode path (B <= 2 tokens): one token at a time through a kernel that holds
 // every x entry to the per-element bound for any x, i.e. to 2^-26 (persistent tcgen05 kernel,
 // one-token form, bf16 x) or 2^-28 (chained kernel, float32 x) of the largest |x| in the K slice
@@ -123,6 +128,47 @@ static fairy2i_status auto_decode(const void* x, fairy2i_dtype xdt, int64_t B, i
       const fairy2i_status st = fairy2i_wl_matmul_chain(&c, 1, T, 0, nullptr, 0, s);
       if (st != FAIRY2I_OK) return st;
     }
+  }
+  *handled = true;
+  return FAIRY2I_OK;
+}
+
+// B tokens of one call (a group of `count` linears) through the chained kernel, in launches of
+// up to 4 tokens (each a block of consecutive rows of x and y): the skinny-batch decode. The
+// decoded signs of every unit feed the MMAs of all tokens of a launch; each x entry is held to
+// 2^-28 of the largest |x| of its token in the CTA's K slice, so the per-element bound holds for
+// any x. *handled = false (nothing launched) outside the kernel's limits (T <= 4,
+// in_features <= 24576, x 16-byte aligned).
+static fairy2i_status chain_tokens(const void* x, fairy2i_dtype xdt, int64_t B,
+                                   int64_t in_features, int64_t ldx, int count,
+                                   const uint32_t* const* codes, const float* const* scales,
+                                   int64_t out_features, int T, float* const* y, int64_t ldy,
+                                   cudaStream_t s, bool* handled) {
+  *handled = false;
+  const int64_t esz = xdt == FAIRY2I_BF16 ? 2 : 4;
+  if (T > 4 || in_features > 24576 || !aligned(x, 16)) return FAIRY2I_OK;
+  for (int64_t b0 = 0; b0 < B;) {
+    int nb = (int)(B - b0 >= 4 ? 4 : B - b0);
+    fairy2i_chain_call c = {};
+    c.x = static_cast<const char*>(x) + b0 * ldx * esz;
+    c.xdt = xdt;
+    c.count = count;
+    c.in_features = in_features;
+    c.out_features = out_features;
+    for (int g = 0; g < count; ++g) {
+      c.codes[g] = codes[g];
+      c.scales[g] = scales[g];
+      c.y[g] = y[g] + b0 * ldy;
+    }
+    fairy2i_status st;
+    for (;;) {   // fewer tokens per launch where the B tiles of nb do not fit
+      st = launch_wl_chain(&c, 1, T, 0, nullptr, s, nb, ldx, ldy);
+      if (st != FAIRY2I_ERR_INVALID_ARG || nb == 1) break;
+      --nb;
+    }
+    if (st == FAIRY2I_ERR_INVALID_ARG && b0 == 0) return FAIRY2I_OK;
+    if (st != FAIRY2I_OK) return st;
+    b0 += nb;
   }
   *handled = true;
   return FAIRY2I_OK;
@@ -203,6 +249,11 @@ fairy2i_status fairy2i_wl_matmul_path(const void* x, fairy2i_dtype xdt, int64_t 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   bool handled = false;
   fairy2i_status st = FAIRY2I_OK;
+  if (path == 0 && B >= 2 && B <= kSkinnyMaxTokens) {   // skinny batch: chained kernel
+    st = chain_tokens(x, xdt, B, in_features, ldx, 1, &codes, &scales, out_features, T, &y, ldy,
+                      s, &handled);
+    if (handled || st != FAIRY2I_OK) return st;
+  }
   if (path == 3 || (path == 0 && B > 2)) {   // tcgen05 prefill GEMM
     st = launch_wl_prefill(x, xdt, B, in_features, ldx, codes, scales, n, m, out_features, wpr, T,
                            y, ldy, s, &handled);
@@ -216,18 +267,11 @@ fairy2i_status fairy2i_wl_matmul_path(const void* x, fairy2i_dtype xdt, int64_t 
     return FAIRY2I_ERR_INVALID_ARG;   // shape or dtype outside the kernel
   }
   if (path == 2) return FAIRY2I_ERR_INVALID_ARG;   // retired
-  if (path == 5) {   // the chained decode kernel on this one call
-    if (B != 1 || ldy < out_features) return FAIRY2I_ERR_INVALID_ARG;
-    fairy2i_chain_call c = {};
-    c.x = x;
-    c.xdt = xdt;
-    c.count = 1;
-    c.in_features = in_features;
-    c.out_features = out_features;
-    c.codes[0] = codes;
-    c.scales[0] = scales;
-    c.y[0] = y;
-    return fairy2i_wl_matmul_chain(&c, 1, T, 0, nullptr, 0, stream);
+  if (path == 5) {   // the chained decode kernel on this one call, up to 4 tokens a launch
+    st = chain_tokens(x, xdt, B, in_features, ldx, 1, &codes, &scales, out_features, T, &y, ldy,
+                      s, &handled);
+    if (handled || st != FAIRY2I_OK) return st;
+    return FAIRY2I_ERR_INVALID_ARG;
   }
   if (path == 0 && B <= 2) {
     st = auto_decode(x, xdt, B, in_features, ldx, 1, &codes, &scales, n, m, out_features, wpr, T,
@@ -271,25 +315,17 @@ fairy2i_status fairy2i_wl_matmul_group_path(const void* x, fairy2i_dtype xdt, in
     if (!aligned(x, 16) || !aligned(codes[g], 16) || !aligned(y[g], 4) || !aligned(scales[g], 4))
       return FAIRY2I_ERR_ALIGNMENT;
   }
-  if (path == 5) {   // the chained decode kernel on this one group
-    if (B != 1) return FAIRY2I_ERR_INVALID_ARG;
-    fairy2i_chain_call c = {};
-    c.x = x;
-    c.xdt = xdt;
-    c.count = count;
-    c.in_features = in_features;
-    c.out_features = out_features;
-    for (int g = 0; g < count; ++g) {
-      c.codes[g] = codes[g];
-      c.scales[g] = scales[g];
-      c.y[g] = y[g];
-    }
-    return fairy2i_wl_matmul_chain(&c, 1, T, 0, nullptr, 0, stream);
-  }
   const int64_t n = (out_features + 1) / 2, m = (in_features + 1) / 2;
   const int64_t wpr = fairy2i_codes_words_per_row(m);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   bool handled = false;
+  if (path == 5 || (path == 0 && B >= 2 && B <= kSkinnyMaxTokens)) {
+    // the chained decode kernel on this one group, up to 4 tokens a launch
+    const fairy2i_status st = chain_tokens(x, xdt, B, in_features, ldx, count, codes, scales,
+                                           out_features, T, y, ldy, s, &handled);
+    if (handled || st != FAIRY2I_OK) return st;
+    if (path == 5) return FAIRY2I_ERR_INVALID_ARG;
+  }
   if (B <= 2 && path == 0) {   // per token, one launch for the whole group
     const fairy2i_status st = auto_decode(x, xdt, B, in_features, ldx, count, codes, scales, n, m,
                                           out_features, wpr, T, y, ldy, s, &handled);

@@ -67,12 +67,10 @@ constexpr int kEpiWarp0 = kIssWarp0 + kIss;   // 17-24: two groups of four
 constexpr int kBThreads = 256;           // the two epilogue groups build the B tiles
 constexpr int kWarps = kEpiWarp0 + 8;
 constexpr int kThreads = kWarps * 32;
-constexpr int kSlots = 12;               // A slots (unit q in slot q % kSlots)
-constexpr int kSetSlots = kSlots / kSets;
 constexpr int kDigits = 14;
 constexpr int kN = 32;                   // MMA N (2 kDigits used)
-constexpr int kColAcc = 0;               // accumulators [buffer], 32 columns each
-constexpr int kColA = 64;                // A slots, 32 columns each
+constexpr int kMaxTok = 4;               // tokens per launch
+constexpr int kColAcc = 0;               // accumulators [buffer][token], 32 columns each
 constexpr int kColSF = 448;              // unit scale factors
 constexpr int kTmemCols = 512;
 constexpr int kSlotCols = 32;
@@ -88,7 +86,13 @@ constexpr int kSmemLimit = 227 * 1024;
 constexpr uint64_t kWaitNs = 1000000000ull;   // 1 s: a pipeline wait is microseconds
 constexpr uint32_t kIdesc = idesc_mxf4_f32(128, kN);
 constexpr int kBarB = 1, kBarG = 2;      // named barriers: B build (256), epilogue group g (128)
-constexpr int kFixedBars = 2 * kSlots + 8 + kIss + 1;   // mbarriers besides the ring's
+// Tensor-memory plan of a launch with nb tokens: accumulators in columns [0, 64 nb), then the A
+// slots (an even number, 32 columns each) up to the scale factors at column 448.
+__host__ __device__ constexpr int acc_cols(int nb) { return 64 * nb; }
+__host__ __device__ constexpr int num_slots(int nb) { return ((kColSF - acc_cols(nb)) / kSlotCols) & ~1; }
+// mbarriers besides the ring's: sfull, sfree per slot; jfull, jfree, gfull, gfree per buffer;
+// fin per issuer; sfready
+__host__ __device__ constexpr int fixed_bars(int nb) { return 2 * num_slots(nb) + 8 + kIss + 1; }
 
 struct Call {
   const void* x;
@@ -105,6 +109,7 @@ struct Call {
   int xf32;       // x is float32 (else bf16)
   int x_pair;     // pairs of x entries may be loaded as one aligned access
   int x_vec;      // groups of eight bf16 entries may be loaded as one 16-byte access
+  int ldx, ldy;   // elements between the tokens of x and of every y
 };
 
 struct Args {
@@ -125,26 +130,29 @@ struct Misc {
   uint32_t tmem;
   int abort;
   unsigned int bprog;     // B tiles built: (build sequence number << 8) | chunks ready
-  float xmax[8];
-  float S, invS;
+  float xmax[kMaxTok][8];
+  float S[kMaxTok], invS[kMaxTok];
   float scl[kMaxGroup][16];
 };
 
 struct Smem {             // byte offsets from the 1024-aligned base
-  int ring, b, xs, red, gather, outp, tab, bar, misc, total;
+  int ring, b, btok, xs, xtok, red, gather, outp, tab, bar, misc, total;
 };
 
-__host__ __device__ inline Smem smem_layout(int nring, int nu_max, int ncalls) {
+// B tiles and bf16 x staging per token (btok, xtok bytes apart), partial outputs per token.
+__host__ __device__ inline Smem smem_layout(int nring, int nu_max, int ncalls, int nb) {
   Smem s;
   s.ring = 0;
   s.b = s.ring + nring * kUnitBytes;
-  s.xs = s.b + ((nu_max * kChunkB + 15) & ~15);
-  s.red = s.xs + 2 * 72 * nu_max * 4;   // bf16 x staging: 64 nu words per part + 4 per 32
+  s.btok = (nu_max * kChunkB + 15) & ~15;
+  s.xs = s.b + nb * s.btok;
+  s.xtok = 2 * 72 * nu_max * 4;         // bf16 x staging: 64 nu words per part + 4 per 32
+  s.red = s.xs + nb * s.xtok;
   s.gather = s.red + 2 * 128 * 2 * 4;
-  s.outp = s.gather + 2 * kMaxCluster * 64 * 4;
-  s.tab = s.outp + 2 * 64 * 4;
+  s.outp = s.gather + 2 * kMaxCluster * 64 * nb * 4;
+  s.tab = s.outp + 2 * 64 * nb * 4;
   s.bar = s.tab + ncalls * (int)sizeof(Tab);
-  s.misc = s.bar + (2 * nring + kFixedBars) * 8;
+  s.misc = s.bar + (2 * nring + fixed_bars(nb)) * 8;
   s.total = s.misc + (int)sizeof(Misc) + 1024;   // + alignment slack
   return s;
 }
@@ -334,12 +342,12 @@ __device__ __forceinline__ void decode_chunk(const uint32_t (&w)[8], uint32_t se
   }
 }
 
-// Two consecutive x entries k, k + 1 of part p (zero past the part's end): float32 x as floats,
-// bf16 x as one word (entry k in the low half). Plain loads: x may be an output of the previous
-// call, made visible by the completion counter's acquire.
-__device__ __forceinline__ float2 load_x_pair_f32(const Call& C, int p, int k) {
+// Two consecutive x entries k, k + 1 of part p of token b (zero past the part's end): float32 x
+// as floats, bf16 x as one word (entry k in the low half). Plain loads: x may be an output of
+// the previous call, made visible by the completion counter's acquire.
+__device__ __forceinline__ float2 load_x_pair_f32(const Call& C, int b, int p, int k) {
   const int lim = p ? C.in_features - C.m : C.m;
-  const float* x = static_cast<const float*>(C.x) + p * C.m;
+  const float* x = static_cast<const float*>(C.x) + (size_t)b * C.ldx + p * C.m;
   float2 v = make_float2(0.f, 0.f);
   if (C.x_pair && k + 1 < lim) {
     v = *reinterpret_cast<const float2*>(x + k);
@@ -349,19 +357,15 @@ __device__ __forceinline__ float2 load_x_pair_f32(const Call& C, int p, int k) {
   }
   return v;
 }
-__device__ __forceinline__ uint32_t load_x_pair_bf16(const Call& C, int p, int k) {
-  const int lim = p ? C.in_features - C.m : C.m;
-  const unsigned short* x = static_cast<const unsigned short*>(C.x) + p * C.m;
-  if (C.x_pair && k + 1 < lim) return *reinterpret_cast<const unsigned int*>(x + k);
-  const uint32_t lo = k < lim ? (uint32_t)x[k] : 0u;
-  const uint32_t hi = k + 1 < lim ? (uint32_t)x[k + 1] : 0u;
-  return lo | (hi << 16);
-}
 __device__ __forceinline__ float bf_lo(uint32_t v) { return __uint_as_float(v << 16); }
 __device__ __forceinline__ float bf_hi(uint32_t v) { return __uint_as_float(v & 0xffff0000u); }
 
-template <int T>
+template <int T, int NB>
 __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_constant__ Args a) {
+  constexpr int kColA = acc_cols(NB);          // A slots, 32 columns each
+  constexpr int kSlots = num_slots(NB);        // unit q in slot q % kSlots
+  constexpr int kSetSlots = kSlots / kSets;
+  static_assert(kSlots >= 2 * kSets && kSlots % kSets == 0, "A slots");
   constexpr int TM = 2 * T;
   constexpr int R = (T == 1) ? 32 : (T == 2 ? 16 : 8);   // rows per row block
   constexpr bool kHalf = R == 8;                          // a job holds half of a 16-row tile
@@ -370,7 +374,7 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
   unsigned char* smem = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int ncalls = a.ncalls, nring = a.nring, ks = a.ks;
-  const Smem L = smem_layout(nring, a.nu_max, ncalls);
+  const Smem L = smem_layout(nring, a.nu_max, ncalls, NB);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L.bar);
   uint64_t* full = bars;                       // [ring slot] codes landed (tx)
   uint64_t* empty = full + nring;              // [ring slot] codes read (4 warps)
@@ -386,8 +390,8 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
   Tab* tab = reinterpret_cast<Tab*>(smem + L.tab);
   volatile int* abort_flag = &misc->abort;
   float* red = reinterpret_cast<float*>(smem + L.red);          // [group][lane][2]
-  float* gather = reinterpret_cast<float*>(smem + L.gather);    // [group][rank][64]
-  float* outp = reinterpret_cast<float*>(smem + L.outp);        // [group][64]
+  float* gather = reinterpret_cast<float*>(smem + L.gather);    // [group][rank][token][64]
+  float* outp = reinterpret_cast<float*>(smem + L.outp);        // [group][token][64]
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int rank = ks > 1 ? (int)cluster_ctarank() : 0;
@@ -407,7 +411,7 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
     tab[c] = t;
   }
   if (warp == 1) {
-    const int nb = 2 * nring + kFixedBars;
+    const int nb = 2 * nring + fixed_bars(NB);
     for (int i = lane; i < nb; i += 32) {
       uint64_t* b = bars + i;
       uint32_t cnt = 1;
@@ -445,8 +449,8 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
     tmem_st32(la + kColSF + 32, ones);
 #pragma unroll
     for (int i = 0; i < 32; ++i) ones[i] = 0u;
-    tmem_st32(la + kColAcc, ones);
-    tmem_st32(la + kColAcc + 32, ones);
+#pragma unroll
+    for (int c = 0; c < acc_cols(NB); c += 32) tmem_st32(la + kColAcc + c, ones);
     tmem_wait_st();
     tc_fence_before();
     __syncwarp();
@@ -589,9 +593,12 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
         (void)mbar_wait_timed(&full[i % nring], (i / nring) & 1, 1000000ull);
     }
   } else if (warp < kEpiWarp0) {
-    // ---- MMA issuers: lane 0 of warp kIssWarp0 + e issues unit v of a job when
-    // (v + r) % kIss == e, r = the units of this CTA before the job; unit q (counted over the
-    // whole chain) sits in A slot q % kSlots ----
+    // ---- MMA issuers: lane 0 of warp kIssWarp0 + e (e < kIssN) issues unit v of a job when
+    // (v + r) % kIssN == e, r = the units of this CTA before the job; unit q (counted over the
+    // whole chain) sits in A slot q % kSlots. An issuer reaches unit q only after unit
+    // q - kIssN was written, hence (kIssN <= kSlots, same decoder set, decoded in order) after
+    // unit q - kSlots: the slot's barrier is never two phases behind its waiter. ----
+    constexpr int kIssN = kIss < kSlots ? kIss : kSlots;
     const int e = warp - kIssWarp0;
     if (lane == 0) {
       const uint32_t b_base = smem_u32(smem + L.b);
@@ -609,17 +616,17 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
         int have = 0;
         for (int k = 0; ok && k < tb.nj; ++k, ++J, qb += U) {
           const int buf = J & 1;
-          // the read-out of job J - 2 (same buffer) is done and the accumulator zeroed
+          // the read-out of job J - 2 (same buffer) is done and its accumulators zeroed
           if (J >= 2) ok = wait_or_abort(&jfree[buf], ((J >> 1) - 1) & 1, abort_flag, a.status);
           if (!ok) break;
           tc_fence_after();
-          const int v0 = (e - qb) & (kIss - 1);
-          if (v0 < U) {
-            const uint32_t d_tmem = tmem + kColAcc + (uint32_t)(buf * 32);
-            const int q0 = qb + v0;
-            int si = q0 % kSlots;
-            uint32_t sph = (uint32_t)(q0 / kSlots) & 1u;
-            for (int v = v0; v < U; v += kIss) {
+          int v0 = (e - qb) % kIssN;
+          if (v0 < 0) v0 += kIssN;
+          if (e < kIssN && v0 < U) {
+            const uint32_t d0 = tmem + kColAcc + (uint32_t)(buf * NB * 32);
+            for (int v = v0, q = qb + v0; v < U; v += kIssN, q += kIssN) {
+              const int si = q % kSlots;
+              const uint32_t sph = (uint32_t)(q / kSlots) & 1u;
               const int need = min(tb.nu, 2 * v + 2);
               if (have < need) {
                 ok = wait_bprog(&misc->bprog, (seq << 8) | (uint32_t)need, abort_flag, a.status);
@@ -632,19 +639,18 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
               tc_fence_after();
               const uint32_t a_slot = tmem + kColA + (uint32_t)(si * kSlotCols);
               const int nm = 2 * min(2, tb.nu - 2 * v);
-              const uint64_t bd = desc0 + (uint64_t)((4 * v * kMmaB) >> 4);
 #pragma unroll
-              for (int jm = 0; jm < 4; ++jm)
-                if (jm < nm)
-                  mma_mxf4_ts(d_tmem, a_slot + jm * 8, bd + (uint64_t)((jm * kMmaB) >> 4), kIdesc,
-                              tmem + kColSF, tmem + kColSF + 16, 1u);
+              for (int b = 0; b < NB; ++b) {
+                // token b's B tiles, btok bytes after token b - 1's (a multiple of 16)
+                const uint64_t bd = desc0 + (uint64_t)((b * L.btok + 4 * v * kMmaB) >> 4);
+#pragma unroll
+                for (int jm = 0; jm < 4; ++jm)
+                  if (jm < nm)
+                    mma_mxf4_ts(d0 + b * 32, a_slot + jm * 8, bd + (uint64_t)((jm * kMmaB) >> 4),
+                                kIdesc, tmem + kColSF, tmem + kColSF + 16, 1u);
+              }
               issued = true;
               mma_commit(&sfree[si]);
-              si += kIss;   // this issuer's next unit: q + kIss (kIss < kSlots)
-              if (si >= kSlots) {
-                si -= kSlots;
-                sph ^= 1u;
-              }
             }
             if (!ok) break;
             mma_commit(&jfull[buf]);
@@ -667,11 +673,12 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
     const int et = bt - grp * 128;                 // 0 .. 127 inside the group
     const int quarter = warp & 3;
     const int Ln = quarter * 32 + lane;
-    // Rows 28-31 of every B tile stay zero.
-    for (int o = bt; o < a.nu_max * 2 * 4 * 2; o += kBThreads) {
-      const int tile = o >> 3, rest = o & 7, nrow = 2 * kDigits + (rest >> 1);
-      *reinterpret_cast<uint4*>(smem + L.b + tile * kMmaB + (nrow >> 3) * 256 + (rest & 1) * 128 +
-                                (nrow & 7) * 16) = make_uint4(0, 0, 0, 0);
+    // Rows 28-31 of every B tile of every token stay zero.
+    for (int o = bt; o < NB * a.nu_max * 2 * 4 * 2; o += kBThreads) {
+      const int tb_ = o / (a.nu_max * 16), oo = o - tb_ * (a.nu_max * 16);
+      const int tile = oo >> 3, rest = oo & 7, nrow = 2 * kDigits + (rest >> 1);
+      *reinterpret_cast<uint4*>(smem + L.b + tb_ * L.btok + tile * kMmaB + (nrow >> 3) * 256 +
+                                (rest & 1) * 128 + (nrow & 7) * 16) = make_uint4(0, 0, 0, 0);
     }
     pdl_wait_primary();   // x may be written, and y read, by the previous kernel
     if (ks > 1) cluster_wait();   // every rank's barriers are initialised
@@ -684,12 +691,14 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
         // While the previous call finishes, warm L2 with this CTA's slice of x: a prefetch
         // returns nothing to the program, so it may precede the dependency wait (L2 is the
         // point of coherence of global memory).
-        if (bt < 2) {
-          const int lim = bt ? C.in_features - C.m : C.m;
+        if (bt < 2 * NB) {
+          const int pp = bt & 1, tk = bt >> 1;
+          const int lim = pp ? C.in_features - C.m : C.m;
           const int k0 = 128 * tb.c0, k1 = min(128 * (tb.c0 + tb.nu), lim);
           if (k1 > k0) {
             const int esz = C.xf32 ? 4 : 2;
-            const uintptr_t b0 = reinterpret_cast<uintptr_t>(C.x) + ((size_t)bt * C.m + k0) * esz;
+            const uintptr_t b0 = reinterpret_cast<uintptr_t>(C.x) +
+                                 ((size_t)tk * C.ldx + (size_t)pp * C.m + k0) * esz;
             const uintptr_t a0 = (b0 + 15) & ~uintptr_t(15);
             const uintptr_t a1 = (b0 + (size_t)(k1 - k0) * esz) & ~uintptr_t(15);
             if (a1 > a0) prefetch_l2_bulk(reinterpret_cast<const void*>(a0), (uint32_t)(a1 - a0));
@@ -699,58 +708,71 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
           if (c > 0 && a.done) (void)wait_counter(a.done + (c - 1), (unsigned)ncl, abort_flag, a.status);
         }
         named_bar_sync(kBarB, kBThreads);
-        // Pass 1: max |x| over the slice; bf16 x is staged in shared memory by 16-byte loads
-        // (word w of a part at w + 4 (w / 32): the pass-2 reads of a warp hit 32 banks), float32
-        // x is read twice from global memory.
+        // Pass 1: max |x| over the slice, per token; bf16 x is staged in shared memory by
+        // 16-byte loads (word w of a part at w + 4 (w / 32): the pass-2 reads of a warp hit 32
+        // banks), float32 x is read twice from global memory.
         const bool f32 = C.xf32 != 0;
         const int nv = 16 * tb.nu;        // groups of eight entries per part
-        uint32_t* xs = reinterpret_cast<uint32_t*>(smem + L.xs);
         const int pw = 72 * a.nu_max;      // staging words per part
-        float mx = 0.f;
-        for (int i = bt; i < 2 * nv; i += kBThreads) {
-          const int p = i >= nv ? 1 : 0, v = i - p * nv;
-          const int lim = p ? C.in_features - C.m : C.m;
-          const int k = 128 * tb.c0 + 8 * v;
-          if (!f32) {
-            const unsigned short* xp = static_cast<const unsigned short*>(C.x) + p * C.m;
-            uint4 q;
-            if (C.x_vec && k + 8 <= lim) {
-              q = *reinterpret_cast<const uint4*>(xp + k);
+        float mx[NB];
+#pragma unroll
+        for (int b = 0; b < NB; ++b) mx[b] = 0.f;
+#pragma unroll
+        for (int b = 0; b < NB; ++b) {
+          uint32_t* xs = reinterpret_cast<uint32_t*>(smem + L.xs + b * L.xtok);
+          for (int i = bt; i < 2 * nv; i += kBThreads) {
+            const int p = i >= nv ? 1 : 0, v = i - p * nv;
+            const int lim = p ? C.in_features - C.m : C.m;
+            const int k = 128 * tb.c0 + 8 * v;
+            if (!f32) {
+              const unsigned short* xp =
+                  static_cast<const unsigned short*>(C.x) + (size_t)b * C.ldx + p * C.m;
+              uint4 q;
+              if (C.x_vec && k + 8 <= lim) {
+                q = *reinterpret_cast<const uint4*>(xp + k);
+              } else {
+                uint32_t h[8];
+#pragma unroll
+                for (int z = 0; z < 8; ++z) h[z] = k + z < lim ? (uint32_t)xp[k + z] : 0u;
+                q = make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16),
+                               h[6] | (h[7] << 16));
+              }
+              const uint32_t ww[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+              for (int z = 0; z < 4; ++z)
+                mx[b] = fmaxf(mx[b], fmaxf(fabsf(bf_lo(ww[z])), fabsf(bf_hi(ww[z]))));
+              *reinterpret_cast<uint4*>(xs + p * pw + 4 * v + 4 * (v >> 3)) = q;
             } else {
-              uint32_t h[8];
 #pragma unroll
-              for (int z = 0; z < 8; ++z) h[z] = k + z < lim ? (uint32_t)xp[k + z] : 0u;
-              q = make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16),
-                             h[6] | (h[7] << 16));
-            }
-            const uint32_t ww[4] = {q.x, q.y, q.z, q.w};
-#pragma unroll
-            for (int z = 0; z < 4; ++z)
-              mx = fmaxf(mx, fmaxf(fabsf(bf_lo(ww[z])), fabsf(bf_hi(ww[z]))));
-            *reinterpret_cast<uint4*>(xs + p * pw + 4 * v + 4 * (v >> 3)) = q;
-          } else {
-#pragma unroll
-            for (int z = 0; z < 8; z += 2) {
-              const float2 f = load_x_pair_f32(C, p, k + z);
-              mx = fmaxf(mx, fmaxf(fabsf(f.x), fabsf(f.y)));
+              for (int z = 0; z < 8; z += 2) {
+                const float2 f = load_x_pair_f32(C, b, p, k + z);
+                mx[b] = fmaxf(mx[b], fmaxf(fabsf(f.x), fabsf(f.y)));
+              }
             }
           }
         }
 #pragma unroll
-        for (int o = 16; o >= 1; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-        if (lane == 0) misc->xmax[bt >> 5] = mx;
+        for (int b = 0; b < NB; ++b) {
+#pragma unroll
+          for (int o = 16; o >= 1; o >>= 1) mx[b] = fmaxf(mx[b], __shfl_xor_sync(0xffffffffu, mx[b], o));
+          if (lane == 0) misc->xmax[b][bt >> 5] = mx[b];
+        }
         if (bt < C.G * 4 * T) {
           const int gl = bt / (4 * T), idx = bt - gl * 4 * T;
           misc->scl[gl][idx] = C.scales[gl][idx];
         }
         named_bar_sync(kBarB, kBThreads);
-        float xm = misc->xmax[0];
+        // S = 2^(28 - E) for 2^(E-1) <= max|x| < 2^E (per token): every X = rn(|x| S) < 2^28
+        float Sb[NB];
 #pragma unroll
-        for (int w = 1; w < 8; ++w) xm = fmaxf(xm, misc->xmax[w]);
-        // S = 2^(28 - E) for 2^(E-1) <= max|x| < 2^E: every X = rn(|x| S) < 2^28
-        const int ef = (int)((__float_as_uint(xm) >> 23) & 0xffu);
-        const int se = max(1, min(254, 281 - ef));
-        const float S = __uint_as_float((uint32_t)se << 23);
+        for (int b = 0; b < NB; ++b) {
+          float xm = misc->xmax[b][0];
+#pragma unroll
+          for (int w = 1; w < 8; ++w) xm = fmaxf(xm, misc->xmax[b][w]);
+          const int ef = (int)((__float_as_uint(xm) >> 23) & 0xffu);
+          const int se = max(1, min(254, 281 - ef));
+          Sb[b] = __uint_as_float((uint32_t)se << 23);
+        }
         // Pass 2. Task t: lane ln = s' + 4 (tile % 8) of group (tile / 8, pair, part): B column
         // 4 pair + s' of tile (chunk u, MMA hw), rows p 14 + l. Its eight values (nibble n) are
         // codes 2(3-s'), 2(7-s'), 2(3-s')+1, 2(7-s')+1 of words 4 hw + 2 pair and + 1, i.e. the
@@ -759,9 +781,9 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
         // j the nibble j (digits 2 j, 2 j + 1) of every value.
         // Every round of 256 tasks completes eight chunks, which are published at once (MMAs of
         // the first units start while the later chunks are built).
-        if (bt == 0) {
-          misc->S = S;
-          misc->invS = 2.f / S;
+        if (bt < NB) {
+          misc->S[bt] = Sb[bt];
+          misc->invS[bt] = 2.f / Sb[bt];
         }
         const uint32_t seq = (uint32_t)(nbuilt + 1) << 8;
         const int ntask = 128 * ((2 * tb.nu + 7) >> 3);
@@ -769,10 +791,14 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
           const int t = t0 + bt;
           const int ln = t & 31, sp = ln & 3, tile = ((t >> 7) << 3) + (ln >> 2);
           const int pair = (t >> 6) & 1, p = (t >> 5) & 1;
-          if (t < ntask && tile < 2 * tb.nu) {
+#pragma unroll 1
+          for (int b = 0; b < NB; ++b) {
+          if (t >= ntask || tile >= 2 * tb.nu) break;
           const int u = tile >> 1, hw = tile & 1;
+          const float S = Sb[b];
           float2 pv[4];
           if (!f32) {
+            const uint32_t* xs = reinterpret_cast<const uint32_t*>(smem + L.xs + b * L.xtok);
             const int w0 = 64 * u + 32 * hw + 16 * pair + 3 - sp;
 #pragma unroll
             for (int h = 0; h < 4; ++h) {
@@ -783,7 +809,7 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
           } else {
             const int k = 128 * (tb.c0 + u) + 64 * hw + 32 * pair + 2 * (3 - sp);
 #pragma unroll
-            for (int h = 0; h < 4; ++h) pv[h] = load_x_pair_f32(C, p, k + 8 * h);
+            for (int h = 0; h < 4; ++h) pv[h] = load_x_pair_f32(C, b, p, k + 8 * h);
           }
           // nibble n: n = 0: pair 0 lo, 1: pair 1 lo, 2: pair 0 hi, 3: pair 1 hi, 4-7: +16
           const float vals[8] = {pv[0].x, pv[1].x, pv[0].y, pv[1].y,
@@ -795,7 +821,7 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
             sg |= (__float_as_uint(vals[n]) >> 31) << (4 * n + 3);
           }
           transpose_nibbles(X);
-          unsigned char* col = smem + L.b + tile * kMmaB + pair * 128 + sp * 4;
+          unsigned char* col = smem + L.b + b * L.btok + tile * kMmaB + pair * 128 + sp * 4;
 #pragma unroll
           for (int l = 0; l < kDigits; ++l) {
             const uint32_t w = lop3_and_or(X[l >> 1] >> (2 * (l & 1)), 0x33333333u, sg);
@@ -808,7 +834,9 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
           if (bt == 0) st_release_cta(&misc->bprog, seq | (uint32_t)min(tb.nu, (t0 >> 5) + 8));
         }
         ++nbuilt;
-        const float invS = misc->invS;
+        float invS[NB];
+#pragma unroll
+        for (int b = 0; b < NB; ++b) invS[b] = misc->invS[b];
 
         // -------- the jobs of call c: group grp reads out the jobs of its parity --------
         int g = tb.first / C.rbs, rb = tb.first - g * C.rbs;
@@ -818,74 +846,87 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
             const bool got = __all_sync(0xffffffffu,
                                         wait_or_abort(&jfull[grp], jg & 1, abort_flag, a.status));
             tc_fence_after();
-            float vre = 0.f, vim = 0.f;
-            if (got) {
-              // the 28 digit columns (loads of 16 + 8 + 4, one wait), then zeroes for the
-              // job after next
-              const uint32_t ta = tmem + ((uint32_t)(quarter * 32) << 16) + kColAcc +
-                                  (uint32_t)(grp * 32);
-              float d[28];
-              tmem_ld16(ta, *reinterpret_cast<float(*)[16]>(&d[0]));
-              tmem_ld8(ta + 16, &d[16]);
-              tmem_ld4(ta + 24, &d[24]);
-              tmem_wait_ld();
+            float vre[NB], vim[NB];
 #pragma unroll
-              for (int l = 0; l < kDigits; ++l) {
-                const float wgt = (float)(1u << (2 * l));
-                vre = fmaf(d[l], wgt, vre);
-                vim = fmaf(d[kDigits + l], wgt, vim);
+            for (int b = 0; b < NB; ++b) vre[b] = vim[b] = 0.f;
+            if (got) {
+              // per token: the 28 digit columns (loads of 16 + 8 + 4, one wait), then zeroes
+              // for the job after next
+#pragma unroll
+              for (int b = 0; b < NB; ++b) {
+                const uint32_t ta = tmem + ((uint32_t)(quarter * 32) << 16) + kColAcc +
+                                    (uint32_t)((grp * NB + b) * 32);
+                float d[28];
+                tmem_ld16(ta, *reinterpret_cast<float(*)[16]>(&d[0]));
+                tmem_ld8(ta + 16, &d[16]);
+                tmem_ld4(ta + 24, &d[24]);
+                tmem_wait_ld();
+#pragma unroll
+                for (int l = 0; l < kDigits; ++l) {
+                  const float wgt = (float)(1u << (2 * l));
+                  vre[b] = fmaf(d[l], wgt, vre[b]);
+                  vim[b] = fmaf(d[kDigits + l], wgt, vim[b]);
+                }
+                tmem_zero16(ta);
+                tmem_zero16(ta + 16);
               }
-              tmem_zero16(ta);
-              tmem_zero16(ta + 16);
               tmem_wait_st();
             }
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&jfree[grp]);
+            // row r, component comp of token b: sum over the stage-matrices of h P + conj(h) Q
+            // (U) or h conj(P) + conj(h) conj(Q) (W)
             float* rg = red + grp * 256;
-            rg[Ln * 2 + 0] = vre * invS;
-            rg[Ln * 2 + 1] = vim * invS;
-            named_bar_sync(kBarG + grp, 128);
-            // row r, component comp: sum over the stage-matrices of h P + conj(h) Q (U) or
-            // h conj(P) + conj(h) conj(Q) (W)
-            float val = 0.f;
-            if (et < 2 * R) {
-              const int r = et >> 1, comp = et & 1;
+            float val[NB];
 #pragma unroll
-              for (int tm = 0; tm < TM; ++tm) {
-                const float pre = rg[(tm * R + r) * 2], qre = rg[(64 + tm * R + r) * 2];
-                float pim = rg[(tm * R + r) * 2 + 1], qim = rg[(64 + tm * R + r) * 2 + 1];
-                if (tm & 1) {
-                  pim = -pim;
-                  qim = -qim;
+            for (int b = 0; b < NB; ++b) {
+              rg[Ln * 2 + 0] = vre[b] * invS[b];
+              rg[Ln * 2 + 1] = vim[b] * invS[b];
+              named_bar_sync(kBarG + grp, 128);
+              val[b] = 0.f;
+              if (et < 2 * R) {
+                const int r = et >> 1, comp = et & 1;
+#pragma unroll
+                for (int tm = 0; tm < TM; ++tm) {
+                  const float pre = rg[(tm * R + r) * 2], qre = rg[(64 + tm * R + r) * 2];
+                  float pim = rg[(tm * R + r) * 2 + 1], qim = rg[(64 + tm * R + r) * 2 + 1];
+                  if (tm & 1) {
+                    pim = -pim;
+                    qim = -qim;
+                  }
+                  const float hr = 0.5f * misc->scl[g][tm * 2 + 0];
+                  const float hi = 0.5f * misc->scl[g][tm * 2 + 1];
+                  val[b] += comp == 0 ? hr * (pre + qre) - hi * (pim - qim)
+                                      : hr * (pim + qim) + hi * (pre - qre);
                 }
-                const float hr = 0.5f * misc->scl[g][tm * 2 + 0];
-                const float hi = 0.5f * misc->scl[g][tm * 2 + 1];
-                val += comp == 0 ? hr * (pre + qre) - hi * (pim - qim)
-                                 : hr * (pim + qim) + hi * (pre - qre);
               }
+              named_bar_sync(kBarG + grp, 128);   // red is free for the next token or job
             }
-            named_bar_sync(kBarG + grp, 128);   // red is free for the next job
             bool write = rank == 0;
             if (ks > 1) {
+              // partial rows of every token (64 floats each) go to rank 0 in one bulk copy
               if (rank != 0) {
                 const bool fr = jg < 1 ||
                                 __all_sync(0xffffffffu, wait_or_abort(&gfree[grp], (jg - 1) & 1,
                                                                       abort_flag, a.status));
                 const bool ok2 = fr && !*abort_flag;
-                float* op = outp + grp * 64;
-                if (et < 2 * R) op[et] = ok2 ? val : 0.f;
+                float* op = outp + grp * 64 * NB;
+#pragma unroll
+                for (int b = 0; b < NB; ++b)
+                  if (et < 2 * R) op[b * 64 + et] = ok2 ? val[b] : 0.f;
                 fence_proxy_async_smem();
                 named_bar_sync(kBarG + grp, 128);
                 if (et == 0) {
                   const uint32_t g0 =
-                      smem_u32(gather) + (uint32_t)((grp * kMaxCluster + rank) * 64) * 4;
-                  bulk_copy_to_cluster(mapa_shared(g0, 0), smem_u32(op), (uint32_t)(2 * R * 4),
+                      smem_u32(gather) + (uint32_t)((grp * kMaxCluster + rank) * 64 * NB) * 4;
+                  bulk_copy_to_cluster(mapa_shared(g0, 0), smem_u32(op), (uint32_t)(64 * NB * 4),
                                        mapa_shared(smem_u32(&gfull[grp]), 0));
                   bulk_commit_wait_read();
                 }
               } else {
-                if (et == 0) mbar_arrive_expect_tx(&gfull[grp], (uint32_t)((ks - 1) * 2 * R * 4));
+                if (et == 0)
+                  mbar_arrive_expect_tx(&gfull[grp], (uint32_t)((ks - 1) * 64 * NB * 4));
                 const bool got2 =
                     __all_sync(0xffffffffu, mbar_wait_cluster_poll(&gfull[grp], jg & 1, kWaitNs)) &&
                     !*abort_flag;
@@ -897,7 +938,9 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
                   write = false;
                 } else if (et < 2 * R) {
                   for (int r2 = 1; r2 < ks; ++r2)
-                    val += gather[(grp * kMaxCluster + r2) * 64 + et];
+#pragma unroll
+                    for (int b = 0; b < NB; ++b)
+                      val[b] += gather[((grp * kMaxCluster + r2) * NB + b) * 64 + et];
                 }
                 named_bar_sync(kBarG + grp, 128);   // every read of gather[grp] is done
                 // Rank r waits for this release only before this group's next job, so the last
@@ -910,9 +953,12 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
               const int r = et >> 1, comp = et & 1;
               const int jr = rb * R + r;
               if (jr < C.n) {
-                float* yg = C.y[g];
-                if (comp == 0) yg[jr] = val;
-                else if (C.n + jr < C.out_features) yg[C.n + jr] = val;
+#pragma unroll
+                for (int b = 0; b < NB; ++b) {
+                  float* yg = C.y[g] + (size_t)b * C.ldy;
+                  if (comp == 0) yg[jr] = val[b];
+                  else if (C.n + jr < C.out_features) yg[C.n + jr] = val[b];
+                }
               }
             }
           }
@@ -942,9 +988,9 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
   if (warp == 0) tmem_dealloc(tmem, kTmemCols);
 }
 
-template <int T>
+template <int T, int NB>
 fairy2i_status launch(const Args& a, int grid, int smem, cudaStream_t stream) {
-  auto kern = wl_chain_kernel<T>;
+  auto kern = wl_chain_kernel<T, NB>;
   static std::atomic<uint64_t> smem_set{0};
   if (!smem_attr_once(kern, kSmemLimit, smem_set)) return FAIRY2I_ERR_CUDA;
   cudaLaunchConfig_t cfg = {};
@@ -966,9 +1012,9 @@ fairy2i_status launch(const Args& a, int grid, int smem, cudaStream_t stream) {
 }
 
 // Clusters of `ks` CTAs (one per SM) that can be resident at once on the device (0 if none).
-template <int T>
+template <int T, int NB>
 int max_clusters(int ks) {
-  auto kern = wl_chain_kernel<T>;
+  auto kern = wl_chain_kernel<T, NB>;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemLimit) !=
       cudaSuccess)
     return 0;
@@ -991,29 +1037,55 @@ int max_clusters(int ks) {
   return n;
 }
 
+// Tokens per launch the kernel is built for: 1 to 4.
+inline int tok_index(int nb) { return nb - 1; }
+
+template <int NB>
+int max_clusters_t(int T, int ks) {
+  switch (T) {
+    case 1: return max_clusters<1, NB>(ks);
+    case 2: return max_clusters<2, NB>(ks);
+    case 3: return max_clusters<3, NB>(ks);
+    case 4: return max_clusters<4, NB>(ks);
+  }
+  return 0;
+}
+
+template <int NB>
+fairy2i_status launch_t(int T, const Args& a, int grid, int smem, cudaStream_t stream) {
+  switch (T) {
+    case 1: return launch<1, NB>(a, grid, smem, stream);
+    case 2: return launch<2, NB>(a, grid, smem, stream);
+    case 3: return launch<3, NB>(a, grid, smem, stream);
+    case 4: return launch<4, NB>(a, grid, smem, stream);
+  }
+  return FAIRY2I_ERR_INVALID_ARG;
+}
+
 }  // namespace ch
 
 namespace {
 std::mutex g_ch_mu;
-int g_ch_clusters[64][4][4];   // [device][ks index][T - 1] resident clusters, -1 = unknown
+int g_ch_clusters[64][4][4][4];   // [device][ks index][T - 1][tokens - 1], -1 = unknown
 bool g_ch_init[64];
 }  // namespace
 
-static int ch_resident_clusters(int dev, int ks_idx, int T) {
+static int ch_resident_clusters(int dev, int ks_idx, int T, int nb) {
   std::lock_guard<std::mutex> lock(g_ch_mu);
   if (!g_ch_init[dev]) {
     for (int i = 0; i < 4; ++i)
-      for (int t = 0; t < 4; ++t) g_ch_clusters[dev][i][t] = -1;
+      for (int t = 0; t < 4; ++t)
+        for (int b = 0; b < 4; ++b) g_ch_clusters[dev][i][t][b] = -1;
     g_ch_init[dev] = true;
   }
-  int& v = g_ch_clusters[dev][ks_idx][T - 1];
+  int& v = g_ch_clusters[dev][ks_idx][T - 1][ch::tok_index(nb)];
   if (v < 0) {
     const int ks = 1 << ks_idx;
-    switch (T) {
-      case 1: v = ch::max_clusters<1>(ks); break;
-      case 2: v = ch::max_clusters<2>(ks); break;
-      case 3: v = ch::max_clusters<3>(ks); break;
-      case 4: v = ch::max_clusters<4>(ks); break;
+    switch (nb) {
+      case 1: v = ch::max_clusters_t<1>(T, ks); break;
+      case 2: v = ch::max_clusters_t<2>(T, ks); break;
+      case 3: v = ch::max_clusters_t<3>(T, ks); break;
+      case 4: v = ch::max_clusters_t<4>(T, ks); break;
       default: v = 0;
     }
   }
@@ -1022,13 +1094,19 @@ static int ch_resident_clusters(int dev, int ks_idx, int T) {
 
 int chain_max_calls() { return ch::kMaxCalls; }
 
-// Checks the calls against the kernel's limits (one token, x float32 or bf16, T <= 4,
-// in_features <= 24576) and launches. `done` holds ncalls zeroed counters (unused for one call);
-// cluster_size 0 picks the cluster size, else 1, 2, 4 or 8.
+// Checks the calls against the kernel's limits (nb = 1 to 4 tokens per call, x float32 or
+// bf16, T <= 4, in_features <= 24576) and launches. Token b of call c reads x + b ldx and writes
+// y[g] + b ldy (elements; ignored for nb = 1). `done` holds ncalls zeroed counters (unused for
+// one call); cluster_size 0 picks the cluster size, else 1, 2, 4 or 8.
 fairy2i_status launch_wl_chain(const fairy2i_chain_call* calls, int ncalls, int T,
-                               int cluster_size, unsigned int* done, cudaStream_t stream) {
+                               int cluster_size, unsigned int* done, cudaStream_t stream, int nb,
+                               int64_t ldx, int64_t ldy) {
   using namespace ch;
   if (ncalls < 1 || ncalls > kMaxCalls || T < 1 || T > 4) return FAIRY2I_ERR_INVALID_ARG;
+  if (nb < 1 || nb > kMaxTok) return FAIRY2I_ERR_INVALID_ARG;
+  if (nb == 1) ldx = ldy = 0;
+  if (ldx < 0 || ldy < 0 || ldx > (int64_t(1) << 30) || ldy > (int64_t(1) << 30))
+    return FAIRY2I_ERR_INVALID_ARG;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return FAIRY2I_ERR_CUDA;
   int sms = 0;
@@ -1043,16 +1121,20 @@ fairy2i_status launch_wl_chain(const fairy2i_chain_call* calls, int ncalls, int 
     nch_max = std::max(nch_max, nch);
   }
   if (nch_max > 8 * kMaxNu || nch_max > 192) return FAIRY2I_ERR_INVALID_ARG;
-  // Cluster size: every rank needs a chunk and at most kMaxNu of them; among the sizes that
+  // Cluster size: every rank needs a chunk and at most kMaxNu of them, and the B tiles of nb
+  // tokens (with a ring of at least four units) must fit in shared memory; among the sizes that
   // fit, the automatic choice minimises an estimate of the busiest cluster's time per call:
-  // jobs x (units + an epilogue of about half a unit) + a quarter unit of B tiles per chunk.
+  // jobs x (units + an epilogue of about half a unit) + a quarter unit of B tiles per chunk,
+  // the MMA and B-tile terms growing with the tokens.
   int best_ks = 0, best_ncl = 0;
   double best_cost = 0.0;
   for (int ki = 0; ki < 4; ++ki) {
     const int ks = 1 << ki;
     if (cluster_size != 0 && ks != cluster_size) continue;
-    if (nch_min < ks || (nch_max + ks - 1) / ks > kMaxNu) continue;
-    const int ncl = std::min(ch_resident_clusters(dev, ki, T), sms / ks);
+    const int nu_max = (nch_max + ks - 1) / ks;
+    if (nch_min < ks || nu_max > kMaxNu) continue;
+    if (smem_layout(4, nu_max, ncalls, nb).total > kSmemLimit) continue;
+    const int ncl = std::min(ch_resident_clusters(dev, ki, T, nb), sms / ks);
     if (ncl < 1) continue;
     double cost = 0.0;
     for (int c = 0; c < ncalls; ++c) {
@@ -1060,7 +1142,7 @@ fairy2i_status launch_wl_chain(const fairy2i_chain_call* calls, int ncalls, int 
       const int64_t nch = (m + 127) / 128, nu = (nch + ks - 1) / ks;
       const int64_t jobs = calls[c].count * ((n + R - 1) / R);
       const int64_t per = (jobs + ncl - 1) / ncl;
-      cost += (double)per * (double)((nu + 1) / 2 + 0.5) + 0.25 * (double)nu + 4.0;
+      cost += (double)per * (double)(nb * (nu + 1) / 2 + 0.5) + 0.25 * nb * (double)nu + 4.0;
     }
     if (best_ks == 0 || cost < best_cost) {
       best_cost = cost;
@@ -1101,21 +1183,25 @@ fairy2i_status launch_wl_chain(const fairy2i_chain_call* calls, int ncalls, int 
     C.off = (int)(deal % best_ncl);
     deal += C.jobs;
     C.xf32 = in.xdt == FAIRY2I_F32 ? 1 : 0;
-    C.x_pair = (m % 2 == 0) ? 1 : 0;   // x itself is 16-byte aligned
-    C.x_vec = (m % 8 == 0) ? 1 : 0;
+    C.ldx = (int)ldx;
+    C.ldy = (int)ldy;
+    // wide loads where every token's parts keep their alignment
+    const uintptr_t xa = reinterpret_cast<uintptr_t>(in.x);
+    C.x_pair = (m % 2 == 0 && ldx % 2 == 0 && xa % 8 == 0) ? 1 : 0;
+    C.x_vec = (m % 8 == 0 && ldx % 8 == 0 && xa % 16 == 0) ? 1 : 0;
   }
   // The code ring takes the shared memory the rest leaves.
-  const Smem base = smem_layout(0, a.nu_max, ncalls);
+  const Smem base = smem_layout(0, a.nu_max, ncalls, nb);
   a.nring = std::min(kMaxRing, (kSmemLimit - base.total - 2 * 8) / (kUnitBytes + 16));
   if (a.nring < 4) return FAIRY2I_ERR_INVALID_ARG;
-  const Smem lay = smem_layout(a.nring, a.nu_max, ncalls);
+  const Smem lay = smem_layout(a.nring, a.nu_max, ncalls, nb);
   if (lay.total > kSmemLimit) return FAIRY2I_ERR_INVALID_ARG;
   const int grid = best_ncl * best_ks;
-  switch (T) {
-    case 1: return launch<1>(a, grid, lay.total, stream);
-    case 2: return launch<2>(a, grid, lay.total, stream);
-    case 3: return launch<3>(a, grid, lay.total, stream);
-    case 4: return launch<4>(a, grid, lay.total, stream);
+  switch (nb) {
+    case 1: return launch_t<1>(T, a, grid, lay.total, stream);
+    case 2: return launch_t<2>(T, a, grid, lay.total, stream);
+    case 3: return launch_t<3>(T, a, grid, lay.total, stream);
+    case 4: return launch_t<4>(T, a, grid, lay.total, stream);
   }
   return FAIRY2I_ERR_INVALID_ARG;
 }

@@ -92,7 +92,7 @@ def test_wl_matmul_validation(lib):
     assert call(B=0) == 0                      # empty batch: nothing to do
     assert call(B=-1) == 1 and call(T=0) == 1 and call(path=6) == 1 and call(x=None) == 1
     assert call(path=2) == 1                   # retired
-    assert call(path=5, B=2) == 1 and call(path=5, T=5) == 1   # the chained kernel: one token, T <= 4
+    assert call(path=5, T=5) == 1   # the chained kernel: T <= 4
     assert call(xdt=7) == 4
     assert call(ldx=15) == 2 and call(ldy=15) == 2
     assert call(x=ODD) == 3 and call(codes=ODD) == 3

@@ -232,10 +232,6 @@ def test_chain_repeated_launches_are_deterministic(F):
 def test_chain_rejects_outside_its_domain(F):
     n, m, T = 16, 64, 2
     codes, scales = _random_quantized(n, m, T, seed=71)
-    cd, sc = _upload(codes), torch.from_numpy(scales).to(DEV)
-    with pytest.raises(F.Fairy2iError) as e:     # two tokens
-        F.wl_matmul(synth.outlier_activations(2, 2 * m, seed=1).to(DEV), cd, sc, 2 * n, path=PATH)
-    assert e.value.code == 1
     codes5, scales5 = _random_quantized(n, m, 5, seed=72)
     with pytest.raises(F.Fairy2iError) as e:     # T = 5
         F.wl_matmul(synth.outlier_activations(1, 2 * m, seed=1).to(DEV), _upload(codes5),

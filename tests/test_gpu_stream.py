@@ -164,25 +164,23 @@ def test_stream_rejects_outside_its_domain(F):
     assert F.get_status() == 0
 
 
-def test_automatic_decode_runs_the_one_token_kernel_per_token(F):
-    """The automatic decode path (B <= 2, bf16 x) runs the persistent kernel's one-token form
-    token by token, one launch per token for a whole group: bit for bit the results of explicit
-    one-token path-4 calls (the kernel is deterministic and a token's result does not depend on
-    the other token)."""
+def test_automatic_decode_kernels(F):
+    """The automatic path runs one token (bf16 x) on the persistent kernel's one-token form and
+    2 to 8 tokens on the chained kernel (path 5), one launch for a whole group: bit for bit the
+    results of the explicit paths (every kernel is deterministic for a given launch shape)."""
     out_f, in_f, T = 4096, 4096, 2
     n, m = O.complex_dims(out_f, in_f)
     layers = [_random_quantized(n, m, T, seed=81 + g) for g in range(3)]
     cds = [_upload(c) for c, _ in layers]
     scs = [torch.from_numpy(s).to(DEV) for _, s in layers]
-    x = synth.outlier_activations(2, in_f, seed=83).to(DEV)
-    auto_group = F.wl_matmul_group(x, cds, scs, out_f)
-    auto_single = F.wl_matmul(x, cds[0], scs[0], out_f)
-    for b in range(2):
-        xb = x[b:b + 1].contiguous()
-        per_token = F.wl_matmul_group(xb, cds, scs, out_f, path=PATH)
-        for a, p in zip(auto_group, per_token):
-            assert torch.equal(a[b:b + 1], p)
-        assert torch.equal(auto_single[b:b + 1], F.wl_matmul(xb, cds[0], scs[0], out_f, path=PATH))
+    for B, path in ((1, PATH), (2, 5), (5, 5)):
+        x = synth.outlier_activations(B, in_f, seed=83 + B).to(DEV)
+        auto_group = F.wl_matmul_group(x, cds, scs, out_f)
+        explicit = F.wl_matmul_group(x, cds, scs, out_f, path=path)
+        for a, p in zip(auto_group, explicit):
+            assert torch.equal(a, p)
+        assert torch.equal(F.wl_matmul(x, cds[0], scs[0], out_f),
+                           F.wl_matmul(x, cds[0], scs[0], out_f, path=path))
     assert F.get_status() == 0
 
 
