@@ -223,7 +223,8 @@ fairy2i_status fairy2i_codes_adjoint(const uint32_t* codes, int64_t n, int64_t m
  * (1 <= count <= FAIRY2I_MAX_GROUP). Where the automatic decode path applies (B <= 8, T <= 4,
  * in_features <= 24576) the whole group is one launch per token (B = 1: the persistent tcgen05
  * kernel's one-token form for bf16 x, the chained kernel for float32 x) or per 4 tokens (the
- * chained kernel); otherwise the members run one after the other on the automatic path. Requirements and errors are those of fairy2i_wl_matmul
+ * chained kernel); B > 8 bf16 tokens on the prefill GEMM: one launch holding every member's tiles;
+ * otherwise the members run one after the other on the automatic path. Requirements and errors are those of fairy2i_wl_matmul
  * for every member (checked before anything is enqueued); FAIRY2I_ERR_INVALID_ARG for a count
  * out of range or a null array. Results agree with the separate calls within the
  * float32-accumulation tolerance (a group splits its work over the SMs differently).

@@ -26,6 +26,12 @@ fairy2i_status launch_wl_prefill(const void* x, fairy2i_dtype xdt, int64_t B, in
                                  int64_t ldx, const uint32_t* codes, const float* scales,
                                  int64_t n, int64_t m, int64_t out_features, int64_t wpr, int T,
                                  float* y, int64_t ldy, cudaStream_t stream, bool* handled);
+fairy2i_status launch_wl_prefill_group(const void* x, fairy2i_dtype xdt, int64_t B,
+                                       int64_t in_features, int64_t ldx, int count,
+                                       const uint32_t* const* codes, const float* const* scales,
+                                       int64_t n, int64_t m, int64_t out_features, int64_t wpr,
+                                       int T, float* const* y, int64_t ldy, cudaStream_t stream,
+                                       bool* handled);
 fairy2i_status launch_wl_stream_group(const void* x, fairy2i_dtype xdt, int64_t B,
                                       int64_t in_features, int64_t ldx, int count,
                                       const uint32_t* const* codes, const float* const* scales,
@@ -325,6 +331,12 @@ fairy2i_status fairy2i_wl_matmul_group_path(const void* x, fairy2i_dtype xdt, in
                                            out_features, T, y, ldy, s, &handled);
     if (handled || st != FAIRY2I_OK) return st;
     if (path == 5) return FAIRY2I_ERR_INVALID_ARG;
+  }
+  if (B > kSkinnyMaxTokens && path == 0) {   // one prefill GEMM launch for the whole group
+    const fairy2i_status st = launch_wl_prefill_group(x, xdt, B, in_features, ldx, count, codes,
+                                                      scales, n, m, out_features, wpr, T, y, ldy,
+                                                      s, &handled);
+    if (handled || st != FAIRY2I_OK) return st;
   }
   if (B <= 2 && path == 0) {   // per token, one launch for the whole group
     const fairy2i_status st = auto_decode(x, xdt, B, in_features, ldx, count, codes, scales, n, m,

@@ -76,18 +76,31 @@ constexpr int kSmemBytes = kOffMisc + 64 + 1024;
 static_assert(kSmemBytes > 116 * 1024, "one CTA per SM: it owns all TMEM columns");
 static_assert(kSmemBytes <= 227 * 1024, "shared memory per CTA");
 
+constexpr int kMaxGroup = 4;
+
 struct Args {
-  const uint32_t* codes;
-  const float* scales;
-  float* y;
+  const uint32_t* codes[kMaxGroup];   // linears sharing x (a group), same shape
+  const float* scales[kMaxGroup];
+  float* y[kMaxGroup];
+  int G;            // linears of the group
   unsigned int* status;
   int64_t B, n, out_features, ldy;
   int wpr;          // code words per row (steps of 16 codes)
   int nch;          // 128-code chunks per row (= x stages per tile)
   int row_tiles;    // ceil(n / 16)
-  int row_blocks;   // ceil(n / R)
+  int row_blocks;   // ceil(n / R) per linear
   int tok_tiles;    // ceil(B / 64)
 };
+
+// Tile t (token-tile-major, so that CTAs running together share x in L2): token tile tb, linear g,
+// row block rb.
+__device__ __forceinline__ void tile_coords(const Args& a, int tile, int& g, int& rb, int& tb) {
+  const int per_tok = a.G * a.row_blocks;
+  tb = tile / per_tok;
+  const int rest = tile - tb * per_tok;
+  g = rest / a.row_blocks;
+  rb = rest - g * a.row_blocks;
+}
 
 // Shared-memory descriptor of a K-major operand in the 128-byte swizzle layout: rows of 128 B
 // (64 bf16 of K), 8-row groups 1024 B apart; start address advanced by 32 B per 16-element step.
@@ -136,7 +149,7 @@ __device__ __forceinline__ bool spin_or_abort(uint64_t* bar, uint32_t parity, vo
 
 template <int T>
 __global__ void __launch_bounds__(kThreads, 1)
-    wl_prefill_kernel(const Args a, const __grid_constant__ CUtensorMap xre,
+    wl_prefill_kernel(const __grid_constant__ Args a, const __grid_constant__ CUtensorMap xre,
                       const __grid_constant__ CUtensorMap xim) {
   constexpr int TM = 2 * T;
   constexpr int R = (T == 1) ? 64 : (T == 2 ? 32 : 16);
@@ -160,7 +173,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   float* red = reinterpret_cast<float*>(smem + kOffRed);
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int ntiles = a.row_blocks * a.tok_tiles;
+  const int ntiles = a.G * a.row_blocks * a.tok_tiles;
   const int my_tiles = ntiles > (int)blockIdx.x ? (ntiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
   const int gpt = a.wpr / 4;          // groups per tile (even: 2 per 128-code chunk)
   const int nch = a.nch;              // x stages per tile
@@ -203,7 +216,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     int xq = 0, cq = 0;   // running stage counters over all tiles of this CTA
     for (int it = 0; it < my_tiles && !__shfl_sync(0xffffffffu, *abort_flag, 0); ++it) {
       const int tile = (int)blockIdx.x + it * (int)gridDim.x;
-      const int rb = tile % a.row_blocks, tb = tile / a.row_blocks;
+      int g, rb, tb;
+      tile_coords(a, tile, g, rb, tb);
+      const uint32_t* codes = a.codes[g];
       int ntl = 0;
 #pragma unroll
       for (int rt = 0; rt < RT; ++rt) ntl += (rb * RT + rt < a.row_tiles) ? 1 : 0;
@@ -220,7 +235,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (lane < TM * RT && rt < ntl) {
             const int64_t t16 = (int64_t)tm * a.row_tiles + rb * RT + rt;
             bulk_load(smem + kOffCodes + st * kCStage + lane * kCChunks * 512,
-                      a.codes + (t16 * a.nch + xs) * 128, (uint32_t)(nc * 512), &cfull[st]);
+                      codes + (t16 * a.nch + xs) * 128, (uint32_t)(nc * 512), &cfull[st]);
           }
           ++cq;
         }
@@ -351,8 +366,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int tm = L / R;
     const bool valid = L < TM * R;
     const int t = tm >> 1, mat = tm & 1;
-    const float hr = valid ? 0.5f * __ldg(a.scales + (t * 2 + mat) * 2 + 0) : 0.f;
-    const float hi = valid ? 0.5f * __ldg(a.scales + (t * 2 + mat) * 2 + 1) : 0.f;
     uint32_t eph = 0;                     // phases of the epilogue barrier passed
     // Barrier of the 128 epilogue threads with a bounded wait (false: the kernel aborts).
     auto epi_sync = [&]() -> bool {
@@ -368,7 +381,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     };
     for (int it = 0; it < my_tiles; ++it) {
       const int tile = (int)blockIdx.x + it * (int)gridDim.x;
-      const int rb = tile % a.row_blocks, tb = tile / a.row_blocks;
+      int g, rb, tb;
+      tile_coords(a, tile, g, rb, tb);
+      const float hr = valid ? 0.5f * __ldg(a.scales[g] + (t * 2 + mat) * 2 + 0) : 0.f;
+      const float hi = valid ? 0.5f * __ldg(a.scales[g] + (t * 2 + mat) * 2 + 1) : 0.f;
+      float* const y = a.y[g];
       if (!__all_sync(0xffffffffu, wait_or_abort(accf, it & 1, abort_flag, a.status))) break;
       tc_fence_after();
 #pragma unroll 1
@@ -406,8 +423,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int64_t b = (int64_t)tb * kTok + sb * 16 + (kp >> 1);
         const int64_t j = (int64_t)rb * R + rr;
         if (b < a.B && j < a.n) {
-          if ((kp & 1) == 0) a.y[b * a.ldy + j] = sum;
-          else if (a.n + j < a.out_features) a.y[b * a.ldy + a.n + j] = sum;
+          if ((kp & 1) == 0) y[b * a.ldy + j] = sum;
+          else if (a.n + j < a.out_features) y[b * a.ldy + a.n + j] = sum;
         }
       }
       if (!epi_sync()) break;
@@ -478,14 +495,18 @@ static bool encode_x_map(CUtensorMap* map, const void* base, int64_t width, int6
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// Handles bf16 x with 16-byte aligned rows (ldx % 8 == 0), m % 8 == 0 and T <= 4; anything else
-// is left to the other kernels (*handled = false).
-fairy2i_status launch_wl_prefill(const void* x, fairy2i_dtype xdt, int64_t B, int64_t in_features,
-                                 int64_t ldx, const uint32_t* codes, const float* scales,
-                                 int64_t n, int64_t m, int64_t out_features, int64_t wpr, int T,
-                                 float* y, int64_t ldy, cudaStream_t stream, bool* handled) {
+// Handles bf16 x with 16-byte aligned rows (ldx % 8 == 0), m % 8 == 0 and T <= 4, for a group of
+// 1..4 linears of the same shape on x (one launch: the tiles of every member); anything else is
+// left to the other kernels (*handled = false).
+fairy2i_status launch_wl_prefill_group(const void* x, fairy2i_dtype xdt, int64_t B,
+                                       int64_t in_features, int64_t ldx, int count,
+                                       const uint32_t* const* codes, const float* const* scales,
+                                       int64_t n, int64_t m, int64_t out_features, int64_t wpr,
+                                       int T, float* const* y, int64_t ldy, cudaStream_t stream,
+                                       bool* handled) {
   using namespace pfl;
   *handled = false;
+  if (count < 1 || count > kMaxGroup) return FAIRY2I_OK;
   if (xdt != FAIRY2I_BF16 || T > 4 || (reinterpret_cast<uintptr_t>(x) % 16) != 0 ||
       ldx % 8 != 0 || m % 8 != 0 || B > (int64_t(1) << 30) || wpr > (int64_t(1) << 24))
     return FAIRY2I_OK;
@@ -505,15 +526,19 @@ fairy2i_status launch_wl_prefill(const void* x, fairy2i_dtype xdt, int64_t B, in
     return FAIRY2I_OK;
   const int R = T == 1 ? 64 : (T == 2 ? 32 : 16);
   Args a;
-  a.codes = codes;
-  a.scales = scales;
-  a.y = y;
+  for (int g = 0; g < kMaxGroup; ++g) {
+    const int gg = g < count ? g : 0;
+    a.codes[g] = codes[gg];
+    a.scales[g] = scales[gg];
+    a.y[g] = y[gg];
+  }
+  a.G = count;
   a.status = device_status_word();
   a.B = B; a.n = n; a.out_features = out_features; a.ldy = ldy;
   a.wpr = (int)wpr; a.nch = (int)(wpr / 8); a.row_tiles = (int)((n + 15) / 16);
   a.row_blocks = (int)((n + R - 1) / R);
   a.tok_tiles = (int)((B + kTok - 1) / kTok);
-  const int64_t tiles = (int64_t)a.row_blocks * a.tok_tiles;
+  const int64_t tiles = (int64_t)count * a.row_blocks * a.tok_tiles;
   if (tiles > (int64_t(1) << 30)) return FAIRY2I_OK;
   const int grid = (int)(tiles < g_pfl_sms[dev] ? tiles : g_pfl_sms[dev]);
   *handled = true;
@@ -525,6 +550,14 @@ fairy2i_status launch_wl_prefill(const void* x, fairy2i_dtype xdt, int64_t B, in
   }
   *handled = false;
   return FAIRY2I_OK;
+}
+
+fairy2i_status launch_wl_prefill(const void* x, fairy2i_dtype xdt, int64_t B, int64_t in_features,
+                                 int64_t ldx, const uint32_t* codes, const float* scales,
+                                 int64_t n, int64_t m, int64_t out_features, int64_t wpr, int T,
+                                 float* y, int64_t ldy, cudaStream_t stream, bool* handled) {
+  return launch_wl_prefill_group(x, xdt, B, in_features, ldx, 1, &codes, &scales, n, m,
+                                 out_features, wpr, T, &y, ldy, stream, handled);
 }
 
 }  // namespace fairy2i

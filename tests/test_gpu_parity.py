@@ -251,10 +251,11 @@ def test_wl_matmul_full_size_decode(F, rows, cols, B, seed):
     assert_wl_close(yg, yo, xo, so)
 
 
-@pytest.mark.parametrize("rows,cols,T", [(11008, 4096, 1), (11008, 4096, 2), (4096, 11008, 3)])
+@pytest.mark.parametrize("rows,cols,T", [(11008, 4096, 1), (11008, 4096, 2), (11008, 4096, 3),
+                                         (4096, 11008, 1), (4096, 11008, 2), (4096, 11008, 3)])
 def test_wl_matmul_prefill_sampled(F, rows, cols, T):
-    """2048 tokens through the default path (the tcgen05 prefill GEMM); the oracle computes a
-    sample of 96 output rows for every token."""
+    """2048 tokens through the default path (the tcgen05 prefill GEMM), every (layer, T) pair the
+    benchmark times; the oracle computes a sample of 96 output rows for every token."""
     seed = synth.weight_seed("prefill", 0 if rows > cols else 1)
     co, so = _layer(rows, cols, T, seed)
     B = 2048
@@ -369,7 +370,7 @@ def test_wl_tcgen05_prefill_strided_odd_input(F):
 
 
 def test_wl_auto_path_routes_batches_to_prefill(F):
-    """Above two tokens the default path is the prefill GEMM where it applies: same bits."""
+    """Above eight tokens the default path is the prefill GEMM where it applies: same bits."""
     n, m, T, B = 300, 512, 2, 33
     codes, scales = _random_quantized(n, m, T, seed=23)
     cd = upload_codes(O.pack_codes(codes))
@@ -422,7 +423,10 @@ def test_bounded_wait_latches_timeout_and_context_survives(F):
     (130, 258, 3, 2, 2, torch.bfloat16),      # ragged rows, two tokens
     (4096, 4096, 2, 1, 3, torch.bfloat16),    # the 7B attention projections
     (11008, 4096, 2, 1, 2, torch.bfloat16),   # the 7B gate and up projections
-    (64, 256, 2, 5, 2, torch.bfloat16),       # B > 2: members on the prefill path
+    (64, 256, 2, 5, 2, torch.bfloat16),       # 2 <= B <= 8: the chained kernel, 4 + 1 tokens
+    (64, 256, 2, 12, 2, torch.bfloat16),      # B > 8: one prefill launch for the group
+    (4096, 4096, 2, 64, 3, torch.bfloat16),   # the 7B q/k/v at 64 tokens: 192 tiles, one launch
+    (300, 512, 3, 130, 2, torch.bfloat16),    # ragged rows, three token tiles
     (37, 53, 2, 1, 4, torch.float32),         # fp32 x: members on the general path
 ])
 def test_wl_matmul_group_equals_separate_calls(F, out_f, in_f, T, B, count, dtype):
