@@ -296,16 +296,6 @@ __device__ __forceinline__ void tmem_ld4(uint32_t taddr, float* v) {
   for (int i = 0; i < 4; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-// Zeroes 16 columns of the warp's 32 TMEM lanes.
-__device__ __forceinline__ void tmem_zero16(uint32_t taddr) {
-  const uint32_t z = 0u;
-  asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %1, %1, %1, %1, %1, %1, %1, %1, %1, %1, "
-      "%1, %1, %1, %1, %1};" ::"r"(taddr),
-      "r"(z)
-      : "memory");
-}
-
 // Bounded wait until *counter >= target (acquire); gives up early once any CTA has latched a
 // timeout in the status word.
 __device__ bool wait_counter(const unsigned int* counter, unsigned int target, volatile int* abort,

@@ -84,15 +84,20 @@ constexpr int kLimbs4 = 13;
 
 // Operand form and layout. One token (NB = 1): e2m1 (kind::mxf4), two codes' signs per A byte,
 // one MMA (K = 64) per two code words, x as kLimbs4 base-4 digits in the first 52 of 64 B
-// columns (slot, part, limb); one issuing thread per set. Two tokens: e4m3 (kind::f8f6f4), one MMA (K = 32) per
-// word, x as two e4m3 limbs in 16 B columns (token, limb, slot, part); two issuing threads per
-// set (words 0-3, 4-7). The e2m1 form of two tokens would need 96 accumulator columns per set.
+// columns (slot, part, limb); two issuing threads per set taking alternate units of the set into
+// the set's accumulator (a thread blocks for about 150 cycles on every MMA it issues, so units
+// overlap only across threads; the digit sums are integers, exact in f32, so the order of the two
+// threads' MMAs does not matter; the epilogue zeroes the accumulator after reading it). Two
+// tokens: e4m3 (kind::f8f6f4), one MMA (K = 32) per word, x as two e4m3 limbs in 16 B columns
+// (token, limb, slot, part); two issuing threads per set (words 0-3, 4-7), each into its own
+// accumulator. The e2m1 form of two tokens would need 96 accumulator columns per set.
 template <int NB>
 struct Layout {
   static constexpr bool kF4 = NB == 1;
   static constexpr int kSlots = 3;                          // A slots per set (one unit each)
-  static constexpr int kIss = kF4 ? 1 : 2;                  // MMA-issuing threads per set
-  static constexpr int kNumAcc = kSets * kIss;              // accumulators per job buffer
+  static constexpr int kIss = 2;                            // MMA-issuing threads per set
+  static constexpr int kIssThreads = kSets * kIss;
+  static constexpr int kNumAcc = kF4 ? kSets : kSets * kIss;   // accumulators per job buffer
   static constexpr int kNUsed = kF4 ? 2 * 2 * kLimbs4 : 16; // B columns holding x
   static constexpr int kN = (kNUsed + 15) / 16 * 16;        // MMA N (the rest zero)
   static constexpr int kPart = 128 * NB;                    // floats of one partial (R NB 2)
@@ -116,7 +121,7 @@ struct Layout {
   static constexpr int kOffGather = kOffRed + 128 * 2 * 2 * 4;
   static constexpr int kOffOut = kOffGather + 2 * kMaxCluster * kPart * 4;
   static constexpr int kOffBar = kOffOut + kPart * 4;
-  static constexpr int kNumBars = 2 * kMaxStages + 2 * kSets * kSlots + 2 + 2 + 1 + 2 + 2 + kNumAcc + 1;
+  static constexpr int kNumBars = 2 * kMaxStages + 2 * kSets * kSlots + 2 + 2 + 1 + 2 + 2 + kIssThreads + 1;
   static constexpr int kOffMisc = kOffBar + kNumBars * 8;
   static constexpr int kSmemBytes = kOffMisc + 512 + 1024;   // + alignment slack
   static_assert(kColSF + (kF4 ? 64 : 0) <= kTmemCols, "TMEM columns");
@@ -254,6 +259,8 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
   using Lay = Layout<NB>;
   constexpr bool kF4 = Lay::kF4;
   constexpr int kSlots = Lay::kSlots, kIss = Lay::kIss, kNumAcc = Lay::kNumAcc;
+  constexpr int kIssThreads = Lay::kIssThreads;
+  static_assert(!kF4 || kSlots >= kIss, "an issuer never waits two phases ahead on a slot");
   constexpr int kEpiWarp0 = Lay::kEpiWarp0;
   constexpr int kColSlots = Lay::kColSlots, kSlotCols = Lay::kSlotCols;
   constexpr int kAccStride = Lay::kAccStride, kMmaB = Lay::kMmaB, kChunkB = Lay::kChunkB;
@@ -274,14 +281,14 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
   uint64_t* full = bars;                        // [stage] codes landed        (tx count)
   uint64_t* empty = full + kMaxStages;          // [stage] codes read          (4 warps x nu)
   uint64_t* sfull = empty + kMaxStages;         // [set][slot] A written       (4 warps)
-  uint64_t* sfree = sfull + kSets * kSlots;     // [set][slot] its MMAs done   (kIss commits)
-  uint64_t* jfull = sfree + kSets * kSlots;     // [buffer] job accumulated    (kNumAcc issuers)
+  uint64_t* sfree = sfull + kSets * kSlots;     // [set][slot] its MMAs done   (e2m1: 1, e4m3: kIss commits)
+  uint64_t* jfull = sfree + kSets * kSlots;     // [buffer] job accumulated    (every issuer)
   uint64_t* jfree = jfull + 2;                  // [buffer] job read out       (4 warps)
   uint64_t* bready = jfree + 2;                 // B tiles written             (1 arrival)
   uint64_t* gfull = bready + 1;                 // [buffer] rank 0: partials arrived
   uint64_t* gfree = gfull + 2;                  // [buffer] ranks > 0: rank 0 read the buffer
   uint64_t* fin = gfree + 2;                    // [issuer] abort path
-  uint64_t* sfready = fin + kNumAcc;            // e2m1: scale factors written (4 warps)
+  uint64_t* sfready = fin + kIssThreads;        // e2m1: scale factors written (4 warps)
   Misc* misc = reinterpret_cast<Misc*>(smem + kOffMisc);
   volatile int* abort_flag = &misc->abort;
   float* red = reinterpret_cast<float*>(smem + kOffRed);
@@ -306,8 +313,8 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
       uint32_t cnt = 1;
       if (i >= kMaxStages && i < 2 * kMaxStages) cnt = 4 * nu;                         // empty
       else if (i >= 2 * kMaxStages && i < 2 * kMaxStages + kSets * kSlots) cnt = 4;    // sfull
-      else if (i < 2 * kMaxStages + 2 * kSets * kSlots && i >= 2 * kMaxStages) cnt = kIss;
-      else if (bars + i == jfull || bars + i == jfull + 1) cnt = kNumAcc;
+      else if (i < 2 * kMaxStages + 2 * kSets * kSlots && i >= 2 * kMaxStages) cnt = kF4 ? 1 : kIss;
+      else if (bars + i == jfull || bars + i == jfull + 1) cnt = kIssThreads;
       else if (bars + i == jfree || bars + i == jfree + 1) cnt = 4;
       else if (bars + i == sfready) cnt = 4;
       mbar_init(bars + i, cnt);
@@ -329,6 +336,12 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
     const uint32_t la = tmem + ((uint32_t)(warp * 32) << 16) + Lay::kColSF;
     tmem_st32(la, ones);
     tmem_st32(la + 32, ones);
+    // the shared accumulators start at zero (every MMA adds)
+#pragma unroll
+    for (int i = 0; i < 32; ++i) ones[i] = 0u;
+    const uint32_t lz = tmem + ((uint32_t)(warp * 32) << 16);
+#pragma unroll
+    for (int c = 0; c < kColSlots; c += 32) tmem_st32(lz + c, ones);
     tmem_wait_st();
     tc_fence_before();
     __syncwarp();
@@ -452,8 +465,9 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
         (void)mbar_wait_timed(&full[i % nstages], (i / nstages) & 1, 1000000ull);
     }
   } else if (warp < kEpiWarp0) {
-    // ------ MMA issuers: lane 0 of warp kIssWarp0 + kIss s + e issues words 4e .. 4e+3 of every
-    // unit of set s into its own accumulator of the job's buffer ------
+    // ------ MMA issuers: lane 0 of warp kIssWarp0 + kIss s + e issues, e2m1: the units
+    // l = e, e + kIss, ... of set s into the set's accumulator of the job's buffer; e4m3: words
+    // 4e .. 4e+3 of every unit of set s into its own accumulator ------
     const int ii = warp - kIssWarp0, set = ii / kIss, e = ii % kIss;
     if (lane == 0) {
       const uint32_t b_base = smem_u32(smem + kOffB);
@@ -469,20 +483,23 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
       auto enter_job = [&](int i) {
         if (i >= 2 && ok) ok = wait_or_abort(&jfree[i & 1], ((i >> 1) - 1) & 1, abort_flag, a.status);
       };
-      // Unit q = set + kSets l of the CTA is chunk u of job i, in slot sl of the set for the
-      // (l / kSlots)-th time (phase ph); advanced without divisions, since this thread's loop
-      // overhead adds to every unit.
-      int i = 0, u = set, sl = 0;
-      uint32_t ph = 0;
+      // Unit q = set + kSets l of the CTA is chunk u of job i, in slot sl = l % kSlots of the
+      // set for the (l / kSlots)-th time (phase ph); this thread takes l = l0, l0 + lstep, ...
+      // (e2m1: l0 = e, lstep = kIss; e4m3: every unit). Advanced without divisions in the loop,
+      // since this thread's loop overhead adds to every unit.
+      constexpr int lstep = kF4 ? kIss : 1;
+      const int l0 = kF4 ? e : 0;
+      int i = 0, u = set + kSets * l0, sl = l0 % kSlots;
+      uint32_t ph = (uint32_t)(l0 / kSlots) & 1u;
       while (u >= nu) {
         u -= nu;
         ++i;
       }
       const uint64_t desc0 = smem_desc(b_base, 128, 256);   // + (byte offset >> 4) per tile
-      for (int q = set; ok && q < total; q += kSets) {
+      for (int q = set + kSets * l0; ok && q < total; q += kSets * lstep) {
         if (i != cur) {
           if (cur >= 0) mma_commit(&jfull[cur & 1]);
-          for (int i2 = cur + 1; ok && i2 < i; ++i2) {   // jobs without a unit of this set
+          for (int i2 = cur + 1; ok && i2 < i; ++i2) {   // jobs without a unit of this thread
             enter_job(i2);
             if (ok) mbar_arrive(&jfull[i2 & 1]);
           }
@@ -497,14 +514,15 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
         if (!ok) break;
         tc_fence_after();
         const uint32_t a_slot = tmem + kColSlots + si * kSlotCols;
-        const uint32_t d_tmem = tmem + ((cur & 1) * kNumAcc + ii) * kAccStride;
         const uint64_t bd = desc0 + (uint64_t)((u * kChunkB) >> 4);
-        if constexpr (kF4) {   // MMA j: words 2 j, 2 j + 1 (A columns 8 j ..)
+        if constexpr (kF4) {   // MMA j: words 2 j, 2 j + 1 (A columns 8 j ..); every MMA adds
+          const uint32_t d_tmem = tmem + ((cur & 1) * kNumAcc + set) * kAccStride;
 #pragma unroll
           for (int j = 0; j < 4; ++j)
             mma_mxf4_ts(d_tmem, a_slot + j * 8, bd + (uint64_t)((j * kMmaB) >> 4), Lay::kIdesc,
-                        tmem + Lay::kColSF, tmem + Lay::kColSF + 16, (first && j == 0) ? 0u : 1u);
+                        tmem + Lay::kColSF, tmem + Lay::kColSF + 16, 1u);
         } else {               // MMA w: word w (A columns 8 w ..)
+          const uint32_t d_tmem = tmem + ((cur & 1) * kNumAcc + ii) * kAccStride;
 #pragma unroll
           for (int w4 = 0; w4 < 4; ++w4) {
             const int w = e * 4 + w4;
@@ -515,11 +533,12 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
         first = false;
         issued = true;
         mma_commit(&sfree[si]);
-        if (++sl == kSlots) {
-          sl = 0;
+        sl += lstep;   // lstep < kSlots: at most one wrap
+        if (sl >= kSlots) {
+          sl -= kSlots;
           ph ^= 1u;
         }
-        u += kSets;
+        u += kSets * lstep;
         while (u >= nu) {
           u -= nu;
           ++i;
@@ -534,7 +553,7 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
       }
       // Abort path: the MMAs this thread issued finish before TMEM is released.
       if (issued && *abort_flag) {
-        mma_commit(&fin[ii]);
+        mma_commit(&fin[ii]);   // ii < kIssThreads
         (void)mbar_wait_timed(&fin[ii], 0, kWaitNs);
       }
     }
@@ -810,6 +829,13 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
               for (int k = 0; k < 16; ++k) d[k] += v0[k] + v1[k];
             }
           }
+        }
+      }
+      if constexpr (kF4) {   // zero both sets' accumulators of this buffer for job i + 2
+        if (got) {
+#pragma unroll
+          for (int c = 0; c < kSets * kAccStride; c += 16) tmem_zero16(acc0 + c);
+          tmem_wait_st();
         }
       }
       tc_fence_before();
