@@ -200,13 +200,6 @@ __device__ __forceinline__ bool spin_or_abort(uint64_t* bar, uint32_t parity, vo
   return false;
 }
 
-// (a & m) | (b & ~m) as one LOP3.
-__device__ __forceinline__ uint32_t lop3_sel(uint32_t a, uint32_t b, uint32_t m) {
-  uint32_t d;
-  asm("lop3.b32 %0, %1, %2, %3, 0xE4;" : "=r"(d) : "r"(a), "r"(b), "r"(m));
-  return d;
-}
-
 // Bounded wait with acquire at cluster scope (arrivals and bulk copies of other CTAs): polls
 // with a short sleep, so the thread resumes soon after the phase completes.
 __device__ bool mbar_wait_cluster_poll(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
@@ -224,30 +217,6 @@ __device__ bool mbar_wait_cluster_poll(uint64_t* bar, uint32_t parity, uint64_t 
     if (done) return true;
     if (clock64() - t0 > limit) return false;
     __nanosleep(32);
-  }
-}
-
-// In-register transpose of an 8 x 8 matrix of nibbles: nibble j of w[i] becomes nibble i of
-// w[j]. Three stages of block swaps: 16-bit halves (w[i], w[i+4]) and bytes (w[a], w[a+2]) by
-// byte permutes, nibbles (w[a], w[a+1]) by shifts and bit selects.
-__device__ __forceinline__ void transpose_nibbles(uint32_t (&w)[8]) {
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const uint32_t a = w[i], b = w[i + 4];
-    w[i] = prmt(a, b, 0x5410u);
-    w[i + 4] = prmt(a, b, 0x7632u);
-  }
-#pragma unroll
-  for (int i = 0; i < 8; i += (i % 2 == 1) ? 3 : 1) {
-    const uint32_t a = w[i], b = w[i + 2];
-    w[i] = prmt(a, b, 0x6240u);
-    w[i + 2] = prmt(a, b, 0x7351u);
-  }
-#pragma unroll
-  for (int i = 0; i < 8; i += 2) {
-    const uint32_t a = w[i], b = w[i + 1];
-    w[i] = lop3_sel(a, b << 4, 0x0F0F0F0Fu);        // low nibbles from a, high from b
-    w[i + 1] = lop3_sel(a >> 4, b, 0x0F0F0F0Fu);    // low nibbles from a's high, high from b
   }
 }
 

@@ -635,38 +635,40 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
           // register i of the item: codes 2 i (low half) and 2 i + 1 (high half)
           const uint32_t ev[8] = {xv[j][0].x, xv[j][0].y, xv[j][0].z, xv[j][0].w,
                                   xv[j][1].x, xv[j][1].y, xv[j][1].z, xv[j][1].w};
-          uint32_t xc[16], sg[16];   // X and sign of code c of the word
-#pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            xc[2 * i] = __float2uint_rn(fabsf(bf_lo(ev[i])) * S[0]);
-            xc[2 * i + 1] = __float2uint_rn(fabsf(bf_hi(ev[i])) * S[0]);
-            sg[2 * i] = (ev[i] >> 15) & 1u;
-            sg[2 * i + 1] = ev[i] >> 31;
-          }
           // Row (slot, p, l) of the MMA tile of words 2 (w / 2), + 1, half w % 2: A register s
           // of the word pairs nibble n (n < 4) with sigma, nibble n + 4 with tau of the code at
           // bit q = 4 n + 3 - s of a half (code 2 q, or 2 (q - 8) + 1 for q >= 8). The sigma
           // slot holds digit l of x of that code in nibble n of word s, the tau slot in nibble
-          // n + 4.
+          // n + 4. The codes of words s = 0, 1 (group A) and s = 2, 3 (group B), nibble n of
+          // word s at position 4 (s % 2) + n: X = rn(|x| S) of the eight values, transposed as an
+          // 8 x 8 nibble matrix, gives in word j the nibble j (digits 2 j, 2 j + 1) of every
+          // value, so digit l of all eight values is one shift and one LOP3.
+          constexpr int kOrdA[8] = {6, 14, 7, 15, 4, 12, 5, 13};
+          constexpr int kOrdB[8] = {2, 10, 3, 11, 0, 8, 1, 9};
+          uint32_t XA[8], XB[8], sgA = 0u, sgB = 0u;
+#pragma unroll
+          for (int n = 0; n < 8; ++n) {
+            const uint32_t va = ev[kOrdA[n] >> 1], vb = ev[kOrdB[n] >> 1];
+            const float fa = (kOrdA[n] & 1) ? bf_hi(va) : bf_lo(va);
+            const float fb = (kOrdB[n] & 1) ? bf_hi(vb) : bf_lo(vb);
+            XA[n] = __float2uint_rn(fabsf(fa) * S[0]);
+            XB[n] = __float2uint_rn(fabsf(fb) * S[0]);
+            sgA |= (__float_as_uint(fa) >> 31) << (4 * n + 3);
+            sgB |= (__float_as_uint(fb) >> 31) << (4 * n + 3);
+          }
+          transpose_nibbles(XA);
+          transpose_nibbles(XB);
           unsigned char* tile = smem + kOffB + u * kChunkB + (w >> 1) * kMmaB + (w & 1) * 128;
 #pragma unroll
           for (int l = 0; l < kLimbs4; ++l) {
-            uint32_t ws[4];
-#pragma unroll
-            for (int sh = 0; sh < 4; ++sh) {
-              ws[sh] = 0u;
-#pragma unroll
-              for (int nn = 0; nn < 4; ++nn) {
-                const int q = 4 * nn + 3 - sh;
-                const int c = q < 8 ? 2 * q : 2 * (q - 8) + 1;
-                ws[sh] |= (((xc[c] >> (2 * l)) & 3u) | (sg[c] << 3)) << (4 * nn);
-              }
-            }
+            const uint32_t wa = lop3_and_or(XA[l >> 1] >> (2 * (l & 1)), 0x33333333u, sgA);
+            const uint32_t wb = lop3_and_or(XB[l >> 1] >> (2 * (l & 1)), 0x33333333u, sgB);
+            const uint32_t ws[4] = {wa & 0xffffu, wa >> 16, wb & 0xffffu, wb >> 16};
             const int ns = p * kLimbs4 + l, nt = (2 + p) * kLimbs4 + l;
             *reinterpret_cast<uint4*>(tile + (ns >> 3) * 256 + (ns & 7) * 16) =
                 make_uint4(ws[0], ws[1], ws[2], ws[3]);
             *reinterpret_cast<uint4*>(tile + (nt >> 3) * 256 + (nt & 7) * 16) =
-                make_uint4(ws[0] << 16, ws[1] << 16, ws[2] << 16, ws[3] << 16);
+                make_uint4(wa << 16, wa & 0xffff0000u, wb << 16, wb & 0xffff0000u);
           }
         }
       }
