@@ -84,20 +84,21 @@ constexpr int kLimbs4 = 13;
 
 // Operand form and layout. One token (NB = 1): e2m1 (kind::mxf4), two codes' signs per A byte,
 // one MMA (K = 64) per two code words, x as kLimbs4 base-4 digits in the first 52 of 64 B
-// columns (slot, part, limb); two issuing threads per set taking alternate units of the set into
-// the set's accumulator (a thread blocks for about 150 cycles on every MMA it issues, so units
-// overlap only across threads; the digit sums are integers, exact in f32, so the order of the two
-// threads' MMAs does not matter; the epilogue zeroes the accumulator after reading it). Two
+// columns (slot, part, limb); three issuing threads per set taking every third unit of the set,
+// all six adding into one accumulator per job buffer (a thread blocks for about 150 cycles on
+// every MMA it issues, so units overlap only across threads; the digit sums are integers, exact in
+// f32, so the order of the threads' MMAs does not matter; the epilogue zeroes the accumulator
+// after reading it), which leaves tensor memory for five A slots per set. Two
 // tokens: e4m3 (kind::f8f6f4), one MMA (K = 32) per word, x as two e4m3 limbs in 16 B columns
 // (token, limb, slot, part); two issuing threads per set (words 0-3, 4-7), each into its own
 // accumulator. The e2m1 form of two tokens would need 96 accumulator columns per set.
 template <int NB>
 struct Layout {
   static constexpr bool kF4 = NB == 1;
-  static constexpr int kSlots = 3;                          // A slots per set (one unit each)
-  static constexpr int kIss = 2;                            // MMA-issuing threads per set
+  static constexpr int kSlots = kF4 ? 5 : 3;                // A slots per set (one unit each)
+  static constexpr int kIss = kF4 ? 3 : 2;                  // MMA-issuing threads per set
   static constexpr int kIssThreads = kSets * kIss;
-  static constexpr int kNumAcc = kF4 ? kSets : kSets * kIss;   // accumulators per job buffer
+  static constexpr int kNumAcc = kF4 ? 1 : kSets * kIss;    // accumulators per job buffer
   static constexpr int kNUsed = kF4 ? 2 * 2 * kLimbs4 : 16; // B columns holding x
   static constexpr int kN = (kNUsed + 15) / 16 * 16;        // MMA N (the rest zero)
   static constexpr int kPart = 128 * NB;                    // floats of one partial (R NB 2)
@@ -516,7 +517,7 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
         const uint32_t a_slot = tmem + kColSlots + si * kSlotCols;
         const uint64_t bd = desc0 + (uint64_t)((u * kChunkB) >> 4);
         if constexpr (kF4) {   // MMA j: words 2 j, 2 j + 1 (A columns 8 j ..); every MMA adds
-          const uint32_t d_tmem = tmem + ((cur & 1) * kNumAcc + set) * kAccStride;
+          const uint32_t d_tmem = tmem + (cur & 1) * kAccStride;
 #pragma unroll
           for (int j = 0; j < 4; ++j)
             mma_mxf4_ts(d_tmem, a_slot + j * 8, bd + (uint64_t)((j * kMmaB) >> 4), Lay::kIdesc,
@@ -796,25 +797,17 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
       auto has = [&](int s) { return nu >= kSets || ((s - i * nu) % kSets + kSets) % kSets < nu; };
       const uint32_t acc0 = tmem + ((uint32_t)(quarter * 32) << 16) + buf * kNumAcc * kAccStride;
       if (got) {
-        if constexpr (kF4) {
+        if constexpr (kF4) {   // one accumulator per buffer: 64 columns
 #pragma unroll
           for (int c16 = 0; c16 < Lay::kN / 16; ++c16) {
-            float v[kSets][16];
-#pragma unroll
-            for (int s = 0; s < kSets; ++s) {
-              if (has(s)) {
-                tmem_ld16(acc0 + s * kAccStride + c16 * 16, v[s]);
-              } else {
-#pragma unroll
-                for (int k = 0; k < 16; ++k) v[s][k] = 0.f;
-              }
-            }
+            float v[16];
+            tmem_ld16(acc0 + c16 * 16, v);
             tmem_wait_ld();
 #pragma unroll
             for (int k = 0; k < 16; ++k) {
               const int col = c16 * 16 + k;   // (slot 2 + part) kLimbs4 + limb
               if (col < Lay::kNUsed)
-                d4[col / kLimbs4] = fmaf(v[0][k] + v[1][k], (float)(1u << (2 * (col % kLimbs4))),
+                d4[col / kLimbs4] = fmaf(v[k], (float)(1u << (2 * (col % kLimbs4))),
                                          d4[col / kLimbs4]);
             }
           }
@@ -833,10 +826,10 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
           }
         }
       }
-      if constexpr (kF4) {   // zero both sets' accumulators of this buffer for job i + 2
+      if constexpr (kF4) {   // zero the accumulator of this buffer for job i + 2
         if (got) {
 #pragma unroll
-          for (int c = 0; c < kSets * kAccStride; c += 16) tmem_zero16(acc0 + c);
+          for (int c = 0; c < kAccStride; c += 16) tmem_zero16(acc0 + c);
           tmem_wait_st();
         }
       }
