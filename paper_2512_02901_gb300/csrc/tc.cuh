@@ -233,7 +233,26 @@ __device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr) {
   asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr)
                : "memory");
 }
-// Bounded wait with acquire at cluster scope (for arrivals made by other CTAs).
+// Bounded wait with acquire at cluster scope (arrivals and bulk copies of other CTAs): polls
+// with a short sleep, so the thread resumes soon after the phase completes.
+__device__ __forceinline__ bool mbar_wait_cluster_poll(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
+  const long long t0 = clock64();
+  const long long limit = (long long)(limit_ns * 5 / 2);
+  for (;;) {
+    uint32_t done;
+    asm volatile(
+        "{\n .reg .pred p;\n"
+        " mbarrier.test_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n"
+        " selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(done)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    if (done) return true;
+    if (clock64() - t0 > limit) return false;
+    __nanosleep(32);
+  }
+}
+// Bounded wait with acquire at cluster scope (for arrivals made by other CTAs), suspending.
 __device__ __forceinline__ bool mbar_wait_cluster_timed(uint64_t* bar, uint32_t parity,
                                                         uint64_t limit_ns) {
   const long long t0 = clock64();

@@ -200,26 +200,6 @@ __device__ __forceinline__ bool spin_or_abort(uint64_t* bar, uint32_t parity, vo
   return false;
 }
 
-// Bounded wait with acquire at cluster scope (arrivals and bulk copies of other CTAs): polls
-// with a short sleep, so the thread resumes soon after the phase completes.
-__device__ bool mbar_wait_cluster_poll(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
-  const long long t0 = clock64();
-  const long long limit = (long long)(limit_ns * 5 / 2);
-  for (;;) {
-    uint32_t done;
-    asm volatile(
-        "{\n .reg .pred p;\n"
-        " mbarrier.test_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n"
-        " selp.u32 %0, 1, 0, p;\n}\n"
-        : "=r"(done)
-        : "r"(smem_u32(bar)), "r"(parity)
-        : "memory");
-    if (done) return true;
-    if (clock64() - t0 > limit) return false;
-    __nanosleep(32);
-  }
-}
-
 __device__ __forceinline__ unsigned int ld_acquire_cta(const unsigned int* p) {
   unsigned int v;
   asm volatile("ld.acquire.cta.shared::cta.u32 %0, [%1];" : "=r"(v) : "r"(smem_u32(p)) : "memory");

@@ -914,7 +914,7 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
           // stays alive until those copies have landed.
           if (et == 0) mbar_arrive_expect_tx(&gfull[buf], (uint32_t)((ks - 1) * NV * 4));
           const bool got2 = __all_sync(0xffffffffu,
-                                       mbar_wait_cluster_timed(&gfull[buf], (i >> 1) & 1, kWaitNs)) &&
+                                       mbar_wait_cluster_poll(&gfull[buf], (i >> 1) & 1, kWaitNs)) &&
                             !*abort_flag;
           if (!got2) {
             if (!*abort_flag) {
