@@ -44,17 +44,11 @@ namespace fairy2i {
 
 namespace pfl {
 
-constexpr int kIssWarp = 8;                       // warps 0-7 decode; 8, 9: sigma / tau issuers
-constexpr int kCopyWarp = kIssWarp + 2;
-constexpr int kEpiWarp = kCopyWarp + 1;           // 4 epilogue warps
-constexpr int kThreads = (kEpiWarp + 4) * 32;
-constexpr int kTok = 64;                          // tokens per tile
+constexpr int kIssWarp = 8;                       // warps 0-7 decode, then the MMA issuers
 constexpr int kG = 4;                             // A ring: groups of 64 codes (4 steps)
-constexpr int kColD = 0;                          // sigma accumulator: columns 0-127, tau 128-255
+constexpr int kColD = 0;                          // accumulators [plane][issuer], 256 columns
 constexpr int kColA = 256;                        // A ring: 64 columns per group
 constexpr int kTmemCols = 512;
-constexpr int kXSub = 2 * kTok * 128;             // x of 64 codes: 2 parts x 64 tokens x 128 B
-constexpr int kXStage = 2 * kXSub;                // x stage: 128 codes
 constexpr int kXS = 4;                            // x stages
 constexpr int kCChunks = 2;                       // 128-code chunks per code stage (4 groups)
 constexpr int kCS = 3;                            // code stages
@@ -62,19 +56,38 @@ constexpr int kCStage = kCChunks * 8 * 512;       // <= 8 tiles x kCChunks x 512
 constexpr int kGroupsPerCStage = 2 * kCChunks;
 constexpr int kRed = 4 * 16 * 2 * 128;            // floats: [sub-block][16 tokens][2][128 lanes]
 constexpr uint64_t kWaitNs = 1000000000ull;
-// kind::f16, bf16 A and B (format 1), f32 D, K-major, N = 128, M = 128.
-constexpr uint32_t kIdesc =
-    (1u << 4) | (1u << 7) | (1u << 10) | ((128u >> 3) << 17) | ((128u >> 4) << 24);
 
-constexpr int kOffX = 0;                                        // 1024-aligned (swizzle 128 B)
-constexpr int kOffCodes = kOffX + kXS * kXStage;                // 128 KB
-constexpr int kOffRed = kOffCodes + kCS * kCStage;              // + 24 KB
-constexpr int kOffBar = kOffRed + kRed * 4;                     // + 64 KB
-constexpr int kNumBars = 2 * kXS + 2 * kCS + 2 * kG + 5;
-constexpr int kOffMisc = kOffBar + kNumBars * 8;
-constexpr int kSmemBytes = kOffMisc + 64 + 1024;
-static_assert(kSmemBytes > 116 * 1024, "one CTA per SM: it owns all TMEM columns");
-static_assert(kSmemBytes <= 227 * 1024, "shared memory per CTA");
+// Token-tile forms. TOK = 64: N = 128, one issuing thread per sign plane (the tensor pipe is the
+// bound). TOK = 32 (batches of at most 32 tokens): N = 64, two issuing threads per plane taking
+// alternate groups, each into its own accumulator (an issuing thread blocks for about 150 cycles
+// on every MMA, so at the smaller N the issue rate is the bound); the epilogue adds the two in a
+// fixed order, so the result is deterministic.
+template <int TOK>
+struct Cfg {
+  static constexpr int kIssPP = TOK == 32 ? 2 : 1;          // issuing threads per sign plane
+  static constexpr int kIssN = 2 * kIssPP;
+  static constexpr int kCopyWarp = kIssWarp + kIssN;
+  static constexpr int kEpiWarp = kCopyWarp + 1;            // 4 epilogue warps
+  static constexpr int kThreads = (kEpiWarp + 4) * 32;
+  static constexpr int kN = 2 * TOK;                        // B rows: Re x, then Im x
+  static constexpr int kAccCols = kN;                       // columns of one accumulator
+  static constexpr int kSub = TOK / 16;                     // 16-token sub-blocks of a tile
+  static constexpr int kXSub = 2 * TOK * 128;               // x of 64 codes: 2 parts x TOK x 128 B
+  static constexpr int kXStage = 2 * kXSub;                 // x stage: 128 codes
+  // kind::f16, bf16 A and B (format 1), f32 D, K-major, N = kN, M = 128.
+  static constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) |
+                                     ((uint32_t)(kN >> 3) << 17) | ((128u >> 4) << 24);
+  static constexpr int kOffX = 0;                           // 1024-aligned (swizzle 128 B)
+  static constexpr int kOffCodes = kOffX + kXS * kXStage;
+  static constexpr int kOffRed = kOffCodes + kCS * kCStage;
+  static constexpr int kOffBar = kOffRed + kRed * 4;
+  static constexpr int kNumBars = 2 * kXS + 2 * kCS + 2 * kG + 3 + kIssN;
+  static constexpr int kOffMisc = kOffBar + kNumBars * 8;
+  static constexpr int kSmemBytes = kOffMisc + 64 + 1024;
+  static_assert(2 * kIssPP * kAccCols <= kColA, "accumulators");
+  static_assert(kSmemBytes > 116 * 1024, "one CTA per SM: it owns all TMEM columns");
+  static_assert(kSmemBytes <= 227 * 1024, "shared memory per CTA");
+};
 
 constexpr int kMaxGroup = 4;
 
@@ -110,11 +123,11 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t addr) {
 }
 
 __device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
-                                            uint32_t accumulate) {
+                                            uint32_t idesc, uint32_t accumulate) {
   asm volatile(
       "{\n .reg .pred p;\n setp.ne.b32 p, %3, 0;\n"
       " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %4, p;\n}\n" ::"r"(d_tmem),
-      "r"(a_tmem), "l"(b_desc), "r"(accumulate), "r"(kIdesc)
+      "r"(a_tmem), "l"(b_desc), "r"(accumulate), "r"(idesc)
       : "memory");
 }
 
@@ -147,10 +160,15 @@ __device__ __forceinline__ bool spin_or_abort(uint64_t* bar, uint32_t parity, vo
   return false;
 }
 
-template <int T>
-__global__ void __launch_bounds__(kThreads, 1)
+template <int T, int TOK>
+__global__ void __launch_bounds__(Cfg<TOK>::kThreads, 1)
     wl_prefill_kernel(const __grid_constant__ Args a, const __grid_constant__ CUtensorMap xre,
                       const __grid_constant__ CUtensorMap xim) {
+  using C = Cfg<TOK>;
+  constexpr int kIssPP = C::kIssPP, kIssN = C::kIssN, kCopyWarp = C::kCopyWarp;
+  constexpr int kXSub = C::kXSub, kXStage = C::kXStage, kOffX = C::kOffX;
+  constexpr int kOffCodes = C::kOffCodes, kOffRed = C::kOffRed, kOffBar = C::kOffBar;
+  constexpr int kOffMisc = C::kOffMisc;
   constexpr int TM = 2 * T;
   constexpr int R = (T == 1) ? 64 : (T == 2 ? 32 : 16);
   constexpr int RT = R / 16;
@@ -159,15 +177,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kOffBar);
   uint64_t* xfull = bars;                   // x stage landed            (tx)
-  uint64_t* xempty = xfull + kXS;           // x stage consumed          (2 issuer commits)
+  uint64_t* xempty = xfull + kXS;           // x stage consumed          (2 kIssPP issuer commits)
   uint64_t* cfull = xempty + kXS;           // code stage landed         (tx)
   uint64_t* cempty = cfull + kCS;           // code stage read           (8 decoder warps)
   uint64_t* gfull = cempty + kCS;           // group's A stored, x in    (4 warps x 2 pairs)
   uint64_t* gempty = gfull + kG;            // group's A consumed        (2 issuer commits)
-  uint64_t* accf = gempty + kG;             // tile accumulators final   (2 issuer commits)
+  uint64_t* accf = gempty + kG;             // tile accumulators final   (every issuer commits)
   uint64_t* dempty = accf + 1;              // accumulators read out     (4 epilogue warps)
-  uint64_t* fin = dempty + 1;               // [2] issued MMAs complete (end of kernel)
-  uint64_t* ebar = fin + 2;                 // epilogue warps' barrier (128 threads)
+  uint64_t* fin = dempty + 1;               // [issuer] issued MMAs complete (end of kernel)
+  uint64_t* ebar = fin + kIssN;             // epilogue warps' barrier (128 threads)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + kOffMisc);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kOffMisc + 8);
   float* red = reinterpret_cast<float*>(smem + kOffRed);
@@ -181,7 +199,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (tid == 0) {
     for (int i = 0; i < kXS; ++i) {
       mbar_init(&xfull[i], 1);
-      mbar_init(&xempty[i], 2);
+      mbar_init(&xempty[i], 2 * kIssPP);
     }
     for (int i = 0; i < kCS; ++i) {
       mbar_init(&cfull[i], 1);
@@ -191,10 +209,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&gfull[i], 8);
       mbar_init(&gempty[i], 2);
     }
-    mbar_init(accf, 2);
+    mbar_init(accf, kIssN);
     mbar_init(dempty, 4);
-    mbar_init(&fin[0], 1);
-    mbar_init(&fin[1], 1);
+    for (int i = 0; i < kIssN; ++i) mbar_init(&fin[i], 1);
     mbar_init(ebar, 128);
     *abort_flag = 0;
     fence_mbar_init();
@@ -247,10 +264,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) {
           mbar_arrive_expect_tx(&xfull[xst], (uint32_t)kXStage);
           unsigned char* dst = smem + kOffX + xst * kXStage;
-          tma_load_2d(dst, &xre, xs * 128, tb * kTok, &xfull[xst]);
-          tma_load_2d(dst + kXSub / 2, &xim, xs * 128, tb * kTok, &xfull[xst]);
-          tma_load_2d(dst + kXSub, &xre, xs * 128 + 64, tb * kTok, &xfull[xst]);
-          tma_load_2d(dst + kXSub + kXSub / 2, &xim, xs * 128 + 64, tb * kTok, &xfull[xst]);
+          tma_load_2d(dst, &xre, xs * 128, tb * TOK, &xfull[xst]);
+          tma_load_2d(dst + kXSub / 2, &xim, xs * 128, tb * TOK, &xfull[xst]);
+          tma_load_2d(dst + kXSub, &xre, xs * 128 + 64, tb * TOK, &xfull[xst]);
+          tma_load_2d(dst + kXSub + kXSub / 2, &xim, xs * 128 + 64, tb * TOK, &xfull[xst]);
         }
         __syncwarp();
       }
@@ -264,17 +281,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         (void)mbar_wait_timed(&cfull[q % kCS], (q / kCS) & 1, kWaitNs);
     }
     __syncwarp();
-  } else if (warp == kIssWarp || warp == kIssWarp + 1) {
-    // ---------------- MMA issuers: warp 8 the sigma plane, warp 9 the tau plane ----------------
-    const int e = warp - kIssWarp;
+  } else if (warp >= kIssWarp && warp < kIssWarp + kIssN) {
+    // ---- MMA issuers: warp kIssWarp + kIssPP p + e issues, for sign plane p (sigma, tau), the
+    // groups gi = e, e + kIssPP, ... of every tile into its own accumulator ----
+    const int ii = warp - kIssWarp, plane = ii / kIssPP, e = ii % kIssPP;
     if (lane == 0) {
-      int g = 0;   // running group counter
-      const uint32_t dcol = tmem + kColD + e * 128;
-      for (int it = 0; it < my_tiles; ++it) {
+      int gbase = 0;   // groups of the earlier tiles
+      const uint32_t dcol = tmem + kColD + (uint32_t)(ii * C::kAccCols);
+      for (int it = 0; it < my_tiles; ++it, gbase += gpt) {
         if (it > 0 && !spin_or_abort(dempty, (it - 1) & 1, abort_flag, a.status)) break;
         tc_fence_after();
         bool ok = true;
-        for (int gi = 0; gi < gpt; ++gi, ++g) {
+        for (int gi = e; gi < gpt; gi += kIssPP) {
+          const int g = gbase + gi;
           const int slot = g % kG;
           const int xst = (it * nch + (gi >> 1)) % kXS;
           if (!spin_or_abort(&gfull[slot], (g / kG) & 1, abort_flag, a.status)) {
@@ -283,20 +302,21 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           tc_fence_after();
           const uint32_t xaddr = smem_u32(smem + kOffX + xst * kXStage + (gi & 1) * kXSub);
-          const uint32_t acol = tmem + kColA + slot * 64 + e * 8;
+          const uint32_t acol = tmem + kColA + slot * 64 + plane * 8;
 #pragma unroll
           for (int k = 0; k < 4; ++k)   // step k of the group: pair k / 2, step k % 2 of the pair
             mma_bf16_ts(dcol, acol + (k >> 1) * 32 + (k & 1) * 16, smem_desc_sw128(xaddr + k * 32),
-                        (gi > 0 || k > 0) ? 1u : 0u);
+                        C::kIdesc, (gi > e || k > 0) ? 1u : 0u);
           mma_commit(&gempty[slot]);
-          if (gi & 1) mma_commit(&xempty[xst]);
+          // this thread's last group of the x stage (groups 2 s, 2 s + 1)
+          if (kIssPP == 2 || (gi & 1)) mma_commit(&xempty[xst]);
         }
         if (!ok) break;
         mma_commit(accf);
       }
       // Every MMA this thread issued completes before TMEM is released.
-      mma_commit(&fin[e]);
-      (void)mbar_wait_timed(&fin[e], 0, kWaitNs);
+      mma_commit(&fin[ii]);
+      (void)mbar_wait_timed(&fin[ii], 0, kWaitNs);
     }
     __syncwarp();
   } else if (warp < kIssWarp) {
@@ -360,7 +380,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) break;
     }
   } else {
-    // ---------------- warps kEpiWarp .. kEpiWarp + 3: epilogue of each tile ----------------
+    // ---------------- the last four warps: epilogue of each tile ----------------
     const int quarter = warp & 3, L = quarter * 32 + lane;
     const uint32_t t_lane = tmem + ((uint32_t)(quarter * 32) << 16);
     const int tm = L / R;
@@ -389,13 +409,36 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!__all_sync(0xffffffffu, wait_or_abort(accf, it & 1, abort_flag, a.status))) break;
       tc_fence_after();
 #pragma unroll 1
-      for (int sb = 0; sb < 4; ++sb) {   // 16 tokens per sub-block
+      for (int sb = 0; sb < C::kSub; ++sb) {   // 16 tokens per sub-block
+        // accumulator (plane, e): columns [re of the TOK tokens | im]; the issuers of a plane
+        // are added in a fixed order
         float pr[16], pi[16], qr[16], qi[16];
-        tmem_ld16(t_lane + kColD + sb * 16, pr);
-        tmem_ld16(t_lane + kColD + 64 + sb * 16, pi);
-        tmem_ld16(t_lane + kColD + 128 + sb * 16, qr);
-        tmem_ld16(t_lane + kColD + 192 + sb * 16, qi);
+        const uint32_t c0 = t_lane + kColD + sb * 16;
+        constexpr uint32_t kTau = (uint32_t)(kIssPP * C::kAccCols);
+        tmem_ld16(c0, pr);
+        tmem_ld16(c0 + TOK, pi);
+        tmem_ld16(c0 + kTau, qr);
+        tmem_ld16(c0 + kTau + TOK, qi);
         tmem_wait_ld();
+        if constexpr (kIssPP == 2) {
+          float v[16];
+          tmem_ld16(c0 + C::kAccCols, v);
+          tmem_wait_ld();
+#pragma unroll
+          for (int k = 0; k < 16; ++k) pr[k] += v[k];
+          tmem_ld16(c0 + C::kAccCols + TOK, v);
+          tmem_wait_ld();
+#pragma unroll
+          for (int k = 0; k < 16; ++k) pi[k] += v[k];
+          tmem_ld16(c0 + kTau + C::kAccCols, v);
+          tmem_wait_ld();
+#pragma unroll
+          for (int k = 0; k < 16; ++k) qr[k] += v[k];
+          tmem_ld16(c0 + kTau + C::kAccCols + TOK, v);
+          tmem_wait_ld();
+#pragma unroll
+          for (int k = 0; k < 16; ++k) qi[k] += v[k];
+        }
         float* sr = red + sb * (16 * 2 * 128);
 #pragma unroll
         for (int k = 0; k < 16; ++k) {
@@ -413,14 +456,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0) mbar_arrive(dempty);   // the issuers may start the next tile
       if (!epi_sync()) break;
       // sum over the stage-matrices; item = (sub-block, token k, part, row r)
-      for (int item = L; item < 4 * 16 * 2 * R; item += 128) {
+      for (int item = L; item < C::kSub * 16 * 2 * R; item += 128) {
         const int sb = item / (32 * R), rem = item % (32 * R);
         const int rr = rem % R, kp = rem / R;
         const float* sr = red + sb * (16 * 2 * 128) + kp * 128 + rr;
         float sum = 0.f;
 #pragma unroll
         for (int m2 = 0; m2 < TM; ++m2) sum += sr[m2 * R];
-        const int64_t b = (int64_t)tb * kTok + sb * 16 + (kp >> 1);
+        const int64_t b = (int64_t)tb * TOK + sb * 16 + (kp >> 1);
         const int64_t j = (int64_t)rb * R + rr;
         if (b < a.B && j < a.n) {
           if ((kp & 1) == 0) y[b * a.ldy + j] = sum;
@@ -438,16 +481,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) tmem_dealloc(tmem, kTmemCols);
 }
 
-template <int T>
+template <int T, int TOK>
 fairy2i_status launch(const Args& a, const CUtensorMap& xre, const CUtensorMap& xim, int grid,
                       cudaStream_t stream) {
-  auto kern = wl_prefill_kernel<T>;
+  auto kern = wl_prefill_kernel<T, TOK>;
   static std::atomic<uint64_t> smem_set{0};
-  if (!smem_attr_once(kern, kSmemBytes, smem_set)) return FAIRY2I_ERR_CUDA;
+  if (!smem_attr_once(kern, Cfg<TOK>::kSmemBytes, smem_set)) return FAIRY2I_ERR_CUDA;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)grid);
-  cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.blockDim = dim3(Cfg<TOK>::kThreads);
+  cfg.dynamicSmemBytes = Cfg<TOK>::kSmemBytes;
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -481,14 +524,14 @@ static PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
 }
 
 // 2-D map over one part of x: `width` bf16 values per token row (zero beyond), rows `ldx` apart,
-// B rows; box of 64 values x 64 tokens, 128-byte swizzle.
+// B rows; box of 64 values x `tok` tokens, 128-byte swizzle.
 static bool encode_x_map(CUtensorMap* map, const void* base, int64_t width, int64_t B,
-                         int64_t ldx) {
+                         int64_t ldx, int tok) {
   PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
   if (!enc || width < 1) return false;
   const cuuint64_t dims[2] = {(cuuint64_t)width, (cuuint64_t)B};
   const cuuint64_t strides[1] = {(cuuint64_t)ldx * 2};
-  const cuuint32_t box[2] = {64, (cuuint32_t)pfl::kTok};
+  const cuuint32_t box[2] = {64, (cuuint32_t)tok};
   const cuuint32_t estr[2] = {1, 1};
   return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -518,11 +561,14 @@ fairy2i_status launch_wl_prefill_group(const void* x, fairy2i_dtype xdt, int64_t
         cudaDeviceGetAttribute(&g_pfl_sms[dev], cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
       return FAIRY2I_ERR_CUDA;
   }
+  // token tiles of 32 for batches of at most 32 tokens (two issuing threads per sign plane), else
+  // 64
+  const int tok = B <= 32 ? 32 : 64;
   CUtensorMap xre, xim;
   const __nv_bfloat16* xb = reinterpret_cast<const __nv_bfloat16*>(x);
-  if (!encode_x_map(&xre, xb, m, B, ldx)) return FAIRY2I_OK;
+  if (!encode_x_map(&xre, xb, m, B, ldx, tok)) return FAIRY2I_OK;
   const bool has_im = in_features > m;
-  if (!encode_x_map(&xim, has_im ? xb + m : xb, has_im ? in_features - m : 1, B, ldx))
+  if (!encode_x_map(&xim, has_im ? xb + m : xb, has_im ? in_features - m : 1, B, ldx, tok))
     return FAIRY2I_OK;
   const int R = T == 1 ? 64 : (T == 2 ? 32 : 16);
   Args a;
@@ -537,16 +583,20 @@ fairy2i_status launch_wl_prefill_group(const void* x, fairy2i_dtype xdt, int64_t
   a.B = B; a.n = n; a.out_features = out_features; a.ldy = ldy;
   a.wpr = (int)wpr; a.nch = (int)(wpr / 8); a.row_tiles = (int)((n + 15) / 16);
   a.row_blocks = (int)((n + R - 1) / R);
-  a.tok_tiles = (int)((B + kTok - 1) / kTok);
+  a.tok_tiles = (int)((B + tok - 1) / tok);
   const int64_t tiles = (int64_t)count * a.row_blocks * a.tok_tiles;
   if (tiles > (int64_t(1) << 30)) return FAIRY2I_OK;
   const int grid = (int)(tiles < g_pfl_sms[dev] ? tiles : g_pfl_sms[dev]);
   *handled = true;
-  switch (T) {
-    case 1: return launch<1>(a, xre, xim, grid, stream);
-    case 2: return launch<2>(a, xre, xim, grid, stream);
-    case 3: return launch<3>(a, xre, xim, grid, stream);
-    case 4: return launch<4>(a, xre, xim, grid, stream);
+  switch (T * 2 + (tok == 32 ? 1 : 0)) {
+    case 1 * 2: return launch<1, 64>(a, xre, xim, grid, stream);
+    case 2 * 2: return launch<2, 64>(a, xre, xim, grid, stream);
+    case 3 * 2: return launch<3, 64>(a, xre, xim, grid, stream);
+    case 4 * 2: return launch<4, 64>(a, xre, xim, grid, stream);
+    case 1 * 2 + 1: return launch<1, 32>(a, xre, xim, grid, stream);
+    case 2 * 2 + 1: return launch<2, 32>(a, xre, xim, grid, stream);
+    case 3 * 2 + 1: return launch<3, 32>(a, xre, xim, grid, stream);
+    case 4 * 2 + 1: return launch<4, 32>(a, xre, xim, grid, stream);
   }
   *handled = false;
   return FAIRY2I_OK;

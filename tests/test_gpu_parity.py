@@ -321,11 +321,14 @@ def test_retired_path_2_is_rejected(F):
     (64, 256, 1, 64), (64, 256, 2, 3), (37, 144, 2, 70), (64, 256, 3, 130), (64, 256, 4, 64),
     (50, 272, 4, 9), (2, 16, 1, 5), (4096, 4096, 2, 64), (256, 2048, 2, 130), (96, 1024, 3, 200),
     (1000, 4096, 2, 65), (130, 400, 1, 129),
+    # 32-token tiles (B <= 32, two issuing threads per sign plane): full, ragged, the boundary
+    (4096, 4096, 2, 16), (11008, 4096, 2, 32), (4096, 11008, 3, 31), (300, 1024, 4, 17),
+    (64, 256, 1, 33), (2048, 2048, 2, 1),
 ])
 def test_wl_tcgen05_prefill_path(F, out_f, in_f, T, B):
     """The tcgen05 prefill GEMM (path 3): ragged row blocks (R = 64, 32, 16, 16 rows of every
-    stage-matrix for T = 1..4), ragged token tiles (64 tokens), ragged 64-code x stages and
-    128-code chunks, one CTA or many tiles per CTA."""
+    stage-matrix for T = 1..4), ragged token tiles (32 tokens up to a batch of 32, else 64),
+    ragged 64-code x stages and 128-code chunks, one CTA or many tiles per CTA."""
     n, m = O.complex_dims(out_f, in_f)
     codes, scales = _random_quantized(n, m, T, seed=5 * out_f + 3 * in_f + T)
     x = synth.outlier_activations(B, in_f, seed=out_f + in_f + 2)
@@ -334,9 +337,11 @@ def test_wl_tcgen05_prefill_path(F, out_f, in_f, T, B):
     assert_wl_close(yg, O.wl_matmul(xo, codes, scales, out_f), xo, scales)
 
 
+@pytest.mark.parametrize("B", [70, 20])
 @pytest.mark.parametrize("T", [1, 2, 3, 4])
-def test_wl_tcgen05_prefill_all_codes_each_value(F, T):
-    """Every code value at every word position of every stage-matrix lane block, 70 tokens."""
+def test_wl_tcgen05_prefill_all_codes_each_value(F, T, B):
+    """Every code value at every word position of every stage-matrix lane block, 70 tokens (64-token
+    tiles) and 20 (32-token tiles)."""
     n, m = 40, 384
     codes = np.zeros((T, 2, n, m), dtype=np.uint8)
     for t in range(T):
@@ -345,7 +350,7 @@ def test_wl_tcgen05_prefill_all_codes_each_value(F, T):
             codes[t, 1, j] = (np.arange(m) // 16 + 3 * j + t) % 4
     g = np.random.default_rng(10 + T)
     scales = (0.01 + 0.02 * g.random((T, 2, 2))).astype(np.float32)
-    x = synth.outlier_activations(70, 2 * m, seed=17 + T)
+    x = synth.outlier_activations(B, 2 * m, seed=17 + T)
     yg = _run_wl(F, x, codes, scales, 2 * n, path=3)
     xo = x.float().numpy()
     assert_wl_close(yg, O.wl_matmul(xo, codes, scales, 2 * n), xo, scales)
