@@ -500,7 +500,8 @@ def run_batches(F, linears, dev, args):
             rec["us_per_layer"] = round(ms * 1e3 / len(linears), 2)
         rec["path"] = ("persistent tcgen05, one-token form" if B == 1 else
                        "chained tcgen05, up to 4 tokens per launch" if B <= 8 else
-                       "tcgen05 GEMM (64-token tiles)")
+                       "tcgen05 GEMM (%d-token tiles; K split over CTA pairs where the "
+                       "tiles fill the SMs poorly)" % (32 if B <= 32 else 64))
         out.append(rec)
         del calls, x_all, y_all
     torch.cuda.empty_cache()

@@ -126,8 +126,7 @@ __device__ __forceinline__ bool wait_b(uint64_t* bar, uint32_t parity, volatile 
 __global__ void __launch_bounds__(kThreads, 1) ste_gemm_kernel(
     const GArgs a, const __grid_constant__ CUtensorMap gmap, const __grid_constant__ CUtensorMap xmap) {
   extern __shared__ unsigned char smem_raw[];
-  unsigned char* smem = reinterpret_cast<unsigned char*>(
-      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  unsigned char* smem = align_smem_1024(smem_raw);
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + kOffBar);
   uint64_t* empty = full + kStages;
   uint64_t* done = empty + kStages;

@@ -11,6 +11,14 @@ __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
 
+// 1024-byte aligned start of the dynamic shared memory (allocated with 1 KB of slack). Derived
+// from the array by pointer arithmetic, not through an integer, so that the compiler keeps every
+// pointer into it in the shared state space: shared loads and stores, which it knows do not
+// alias global memory.
+__device__ __forceinline__ unsigned char* align_smem_1024(unsigned char* raw) {
+  return raw + ((1024u - (smem_u32(raw) & 1023u)) & 1023u);
+}
+
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count)
                : "memory");

@@ -310,8 +310,7 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
   constexpr bool kHalf = R == 8;                          // a job holds half of a 16-row tile
   static_assert(TM * R <= 64, "lanes per plane");
   extern __shared__ unsigned char smem_raw[];
-  unsigned char* smem = reinterpret_cast<unsigned char*>(
-      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  unsigned char* smem = align_smem_1024(smem_raw);
   const int ncalls = a.ncalls, nring = a.nring, ks = a.ks;
   const Smem L = smem_layout(nring, a.nu_max, ncalls, NB);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L.bar);

@@ -30,6 +30,14 @@
 // 8 and 9 issue the sigma and the tau MMAs; warp 10 copies the codes (bulk copies of whole 16-row
 // tiles) and x (TMA) in; warps 11-14 run the epilogue of each tile (every accumulator column is
 // read out first, so the MMAs of the next tile start before the reduction and the stores).
+//
+// K split over CTA pairs. When the tiles fill the SMs poorly (a few tiles per SM, as at batches of
+// up to 64 tokens: 64 tiles of an attention output projection on 152 SMs) the launch is made of
+// clusters of two CTAs that work the same tile on the two halves of its 128-code chunks. Rank 1
+// sums its partials over the stage-matrices, packs the sums in its reduction buffer and arrives
+// (release, cluster scope) on rank 0's barrier; rank 0 reads them over distributed shared memory
+// and stores its own sum + rank 1's, always in that order, so the result does not depend on
+// timing. Rank 0 returns a credit per tile before rank 1 overwrites the buffer with the next one.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
@@ -81,7 +89,7 @@ struct Cfg {
   static constexpr int kOffCodes = kOffX + kXS * kXStage;
   static constexpr int kOffRed = kOffCodes + kCS * kCStage;
   static constexpr int kOffBar = kOffRed + kRed * 4;
-  static constexpr int kNumBars = 2 * kXS + 2 * kCS + 2 * kG + 3 + kIssN;
+  static constexpr int kNumBars = 2 * kXS + 2 * kCS + 2 * kG + 5 + kIssN;
   static constexpr int kOffMisc = kOffBar + kNumBars * 8;
   static constexpr int kSmemBytes = kOffMisc + 64 + 1024;
   static_assert(2 * kIssPP * kAccCols <= kColA, "accumulators");
@@ -102,11 +110,12 @@ struct Args {
   int nch;          // 128-code chunks per row (= x stages per tile)
   int row_tiles;    // ceil(n / 16)
   int row_blocks;   // ceil(n / R) per linear
-  int tok_tiles;    // ceil(B / 64)
+  int tok_tiles;    // ceil(B / TOK)
+  int split;        // 2: clusters of two CTAs split each tile's chunks; 1: one CTA per tile
 };
 
-// Tile t (token-tile-major, so that CTAs running together share x in L2): token tile tb, linear g,
-// row block rb.
+// Tile t (token-tile-major, so that CTAs (or CTA pairs) running together share x in L2): token
+// tile tb, linear g, row block rb.
 __device__ __forceinline__ void tile_coords(const Args& a, int tile, int& g, int& rb, int& tb) {
   const int per_tok = a.G * a.row_blocks;
   tb = tile / per_tok;
@@ -173,8 +182,7 @@ __global__ void __launch_bounds__(Cfg<TOK>::kThreads, 1)
   constexpr int R = (T == 1) ? 64 : (T == 2 ? 32 : 16);
   constexpr int RT = R / 16;
   extern __shared__ unsigned char smem_raw[];
-  unsigned char* smem = reinterpret_cast<unsigned char*>(
-      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  unsigned char* smem = align_smem_1024(smem_raw);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kOffBar);
   uint64_t* xfull = bars;                   // x stage landed            (tx)
   uint64_t* xempty = xfull + kXS;           // x stage consumed          (2 kIssPP issuer commits)
@@ -186,15 +194,23 @@ __global__ void __launch_bounds__(Cfg<TOK>::kThreads, 1)
   uint64_t* dempty = accf + 1;              // accumulators read out     (4 epilogue warps)
   uint64_t* fin = dempty + 1;               // [issuer] issued MMAs complete (end of kernel)
   uint64_t* ebar = fin + kIssN;             // epilogue warps' barrier (128 threads)
+  uint64_t* pready = ebar + 1;              // K split, rank 0: rank 1's sums stored (128)
+  uint64_t* pfree = pready + 1;             // K split, rank 1: rank 0 has read them (1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + kOffMisc);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kOffMisc + 8);
   float* red = reinterpret_cast<float*>(smem + kOffRed);
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const bool split = a.split == 2;
+  const int rank = split ? (int)cluster_ctarank() : 0;
+  const int unit = split ? (int)blockIdx.x >> 1 : (int)blockIdx.x;     // CTA or CTA pair
+  const int nunits = split ? (int)gridDim.x >> 1 : (int)gridDim.x;
   const int ntiles = a.G * a.row_blocks * a.tok_tiles;
-  const int my_tiles = ntiles > (int)blockIdx.x ? (ntiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
-  const int gpt = a.wpr / 4;          // groups per tile (even: 2 per 128-code chunk)
-  const int nch = a.nch;              // x stages per tile
+  const int my_tiles = ntiles > unit ? (ntiles - 1 - unit) / nunits + 1 : 0;
+  // this CTA's 128-code chunks of every tile: [c0, c0 + nch)
+  const int c0 = (split && rank == 1) ? a.nch / 2 : 0;
+  const int nch = split ? (rank == 0 ? a.nch / 2 : a.nch - a.nch / 2) : a.nch;   // x stages
+  const int gpt = 2 * nch;            // groups per tile (2 per chunk)
 
   if (tid == 0) {
     for (int i = 0; i < kXS; ++i) {
@@ -213,6 +229,8 @@ __global__ void __launch_bounds__(Cfg<TOK>::kThreads, 1)
     mbar_init(dempty, 4);
     for (int i = 0; i < kIssN; ++i) mbar_init(&fin[i], 1);
     mbar_init(ebar, 128);
+    mbar_init(pready, 128);
+    mbar_init(pfree, 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -221,6 +239,7 @@ __global__ void __launch_bounds__(Cfg<TOK>::kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  if (split) cluster_arrive();   // both ranks' barriers initialised (waited before remote use)
   pdl_launch_dependents();
 
   if (warp == kCopyWarp) {
@@ -232,17 +251,17 @@ __global__ void __launch_bounds__(Cfg<TOK>::kThreads, 1)
     pdl_wait_primary();   // x may be written by the previous kernel
     int xq = 0, cq = 0;   // running stage counters over all tiles of this CTA
     for (int it = 0; it < my_tiles && !__shfl_sync(0xffffffffu, *abort_flag, 0); ++it) {
-      const int tile = (int)blockIdx.x + it * (int)gridDim.x;
+      const int tile = unit + it * nunits;
       int g, rb, tb;
       tile_coords(a, tile, g, rb, tb);
       const uint32_t* codes = a.codes[g];
       int ntl = 0;
 #pragma unroll
       for (int rt = 0; rt < RT; ++rt) ntl += (rb * RT + rt < a.row_tiles) ? 1 : 0;
-      for (int xs = 0; xs < nch; ++xs, ++xq) {
-        if (xs % kCChunks == 0) {   // code stage: chunks xs .. xs + kCChunks - 1
+      for (int xs = c0; xs < c0 + nch; ++xs, ++xq) {
+        if ((xs - c0) % kCChunks == 0) {   // code stage: chunks xs .. xs + kCChunks - 1
           const int st = cq % kCS;
-          const int nc = min(kCChunks, nch - xs);
+          const int nc = min(kCChunks, c0 + nch - xs);
           bool ok = cq < kCS ||
                     lane != 0 || wait_or_abort(&cempty[st], ((cq / kCS) - 1) & 1, abort_flag, a.status);
           if (!__all_sync(0xffffffffu, ok)) break;
@@ -399,8 +418,9 @@ __global__ void __launch_bounds__(Cfg<TOK>::kThreads, 1)
       }
       return true;
     };
+    if (split) cluster_wait();   // the peer's barriers are initialised
     for (int it = 0; it < my_tiles; ++it) {
-      const int tile = (int)blockIdx.x + it * (int)gridDim.x;
+      const int tile = unit + it * nunits;
       int g, rb, tb;
       tile_coords(a, tile, g, rb, tb);
       const float hr = valid ? 0.5f * __ldg(a.scales[g] + (t * 2 + mat) * 2 + 0) : 0.f;
@@ -408,6 +428,13 @@ __global__ void __launch_bounds__(Cfg<TOK>::kThreads, 1)
       float* const y = a.y[g];
       if (!__all_sync(0xffffffffu, wait_or_abort(accf, it & 1, abort_flag, a.status))) break;
       tc_fence_after();
+      // K split, rank 1: rank 0 has read the previous tile's partials out of this CTA's buffer
+      if (split && rank == 1 && it > 0 &&
+          !__all_sync(0xffffffffu, mbar_wait_cluster_poll(pfree, (it - 1) & 1, kWaitNs))) {
+        *abort_flag = 1;
+        if (lane == 0) latch_status(a.status, kStatusTimeout);
+        break;
+      }
 #pragma unroll 1
       for (int sb = 0; sb < C::kSub; ++sb) {   // 16 tokens per sub-block
         // accumulator (plane, e): columns [re of the TOK tokens | im]; the issuers of a plane
@@ -455,24 +482,102 @@ __global__ void __launch_bounds__(Cfg<TOK>::kThreads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(dempty);   // the issuers may start the next tile
       if (!epi_sync()) break;
-      // sum over the stage-matrices; item = (sub-block, token k, part, row r)
-      for (int item = L; item < C::kSub * 16 * 2 * R; item += 128) {
-        const int sb = item / (32 * R), rem = item % (32 * R);
-        const int rr = rem % R, kp = rem / R;
-        const float* sr = red + sb * (16 * 2 * 128) + kp * 128 + rr;
-        float sum = 0.f;
+      // Sum over the stage-matrices, four rows at a time. Item = (sub-block, token k, part) at
+      // q = 32 sub-block + 2 k + part, rows 4 rq .. 4 rq + 3 of the row block; thread L takes
+      // rq = L % kRQ and q = L / kRQ + kTP i (kTP a divisor of 32), so every item of a thread
+      // has the same part, its token is (L / kRQ) / 2 + 16 (i / kIPS) + (kTP / 2) (i % kIPS),
+      // and its buffer offset a constant from the thread's first once the loop is unrolled.
+      constexpr int kRQ = R / 4;
+      constexpr int kTP = 128 / kRQ;
+      constexpr int kIPS = 32 / kTP;                // items per sub-block and thread
+      constexpr int kPerThread = C::kSub * kIPS;
+      const int rq = L % kRQ, tp = L / kRQ;
+      const float* red_t = red + tp * 128 + 4 * rq;
+      auto stage_sum = [&](int i) -> float4 {
+        const float* sr = red_t + (i / kIPS) * (16 * 2 * 128) + (i % kIPS) * (kTP * 128);
+        float4 sum = *reinterpret_cast<const float4*>(sr);
 #pragma unroll
-        for (int m2 = 0; m2 < TM; ++m2) sum += sr[m2 * R];
-        const int64_t b = (int64_t)tb * TOK + sb * 16 + (kp >> 1);
-        const int64_t j = (int64_t)rb * R + rr;
-        if (b < a.B && j < a.n) {
-          if ((kp & 1) == 0) y[b * a.ldy + j] = sum;
-          else if (a.n + j < a.out_features) y[b * a.ldy + a.n + j] = sum;
+        for (int m2 = 1; m2 < TM; ++m2) {
+          const float4 v = *reinterpret_cast<const float4*>(sr + m2 * R);
+          sum.x += v.x;
+          sum.y += v.y;
+          sum.z += v.z;
+          sum.w += v.w;
+        }
+        return sum;
+      };
+      if (split && rank == 1) {
+        // K split, rank 1: the sums, packed at red[4 (128 i + L)] once every thread has read
+        // its inputs, then released to rank 0, which reads them
+        float4 part[kPerThread];
+#pragma unroll
+        for (int i = 0; i < kPerThread; ++i) part[i] = stage_sum(i);
+        if (!epi_sync()) break;
+#pragma unroll
+        for (int i = 0; i < kPerThread; ++i) reinterpret_cast<float4*>(red)[128 * i + L] = part[i];
+        mbar_arrive_remote(mapa_shared(smem_u32(pready), 0));
+        if (__shfl_sync(0xffffffffu, *abort_flag, 0)) break;
+        continue;
+      }
+      if (split && !__all_sync(0xffffffffu, mbar_wait_cluster_poll(pready, it & 1, kWaitNs))) {
+        *abort_flag = 1;
+        if (lane == 0) latch_status(a.status, kStatusTimeout);
+        break;
+      }
+      // this CTA's sum, plus (K split) rank 1's, in that order; one 16-byte store per item where
+      // the four outputs exist and are 16-byte aligned, else one store per existing output
+      const int im = tp & 1;
+      const int64_t j = (int64_t)rb * R + 4 * rq;
+      const int64_t b0 = (int64_t)tb * TOK + (tp >> 1);
+      const int64_t nb = a.B - b0;                  // tokens of y from b0 on
+      const int64_t lim = im ? min(a.n, a.out_features - a.n) : a.n;   // rows j < lim exist
+      float* const yt = y + b0 * a.ldy + im * a.n + j;
+      const bool vec = j + 3 < lim && (a.ldy & 3) == 0 && (reinterpret_cast<uintptr_t>(yt) & 15) == 0;
+      const uint32_t peer_red = split ? mapa_shared(smem_u32(red), 1) + 16u * L : 0u;
+      constexpr int kBatch = kPerThread < 4 ? kPerThread : 4;   // rank 1's sums loaded together
+#pragma unroll
+      for (int i0 = 0; i0 < kPerThread; i0 += kBatch) {
+        float4 other[kBatch];
+        if (split) {
+#pragma unroll
+          for (int u = 0; u < kBatch; ++u) other[u] = ld_cluster_f32x4(peer_red + 2048u * (i0 + u));
+        }
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) {
+          const int i = i0 + u;
+          float4 out = stage_sum(i);
+          if (split) {
+            out.x += other[u].x;
+            out.y += other[u].y;
+            out.z += other[u].z;
+            out.w += other[u].w;
+          }
+          const int db = 16 * (i / kIPS) + (kTP / 2) * (i % kIPS);
+          if (db < nb) {
+            float* const yp = yt + db * a.ldy;
+            if (vec) {
+              *reinterpret_cast<float4*>(yp) = out;
+            } else {
+              if (j < lim) yp[0] = out.x;
+              if (j + 1 < lim) yp[1] = out.y;
+              if (j + 2 < lim) yp[2] = out.z;
+              if (j + 3 < lim) yp[3] = out.w;
+            }
+          }
         }
       }
       if (!epi_sync()) break;
+      if (split && L == 0) mbar_arrive_remote(mapa_shared(smem_u32(pfree), 1));
       if (__shfl_sync(0xffffffffu, *abort_flag, 0)) break;
     }
+  }
+
+  // K split: neither CTA exits while the other may still arrive on its barriers (every wait
+  // above is bounded, so every thread of the pair gets here).
+  if (split) {
+    if (warp < C::kEpiWarp) cluster_wait();   // the epilogue warps waited the first phase
+    cluster_arrive();
+    cluster_wait();
   }
 
   tc_fence_before();
@@ -492,13 +597,57 @@ fairy2i_status launch(const Args& a, const CUtensorMap& xre, const CUtensorMap& 
   cfg.blockDim = dim3(Cfg<TOK>::kThreads);
   cfg.dynamicSmemBytes = Cfg<TOK>::kSmemBytes;
   cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = (unsigned)a.split;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = a.split == 2 ? 2 : 1;
   if (cudaLaunchKernelEx(&cfg, kern, a, xre, xim) != cudaSuccess) return FAIRY2I_ERR_CUDA;
   return FAIRY2I_OK;
+}
+
+// CTA pairs (clusters of two) of the kernel that can be resident at once; 0 if none.
+template <int T, int TOK>
+int max_pairs() {
+  auto kern = wl_prefill_kernel<T, TOK>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           Cfg<TOK>::kSmemBytes) != cudaSuccess)
+    return 0;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2 * 256);
+  cfg.blockDim = dim3(Cfg<TOK>::kThreads);
+  cfg.dynamicSmemBytes = Cfg<TOK>::kSmemBytes;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return 0;
+  }
+  return n;
+}
+
+inline int max_pairs_t(int T, int tok) {
+  switch (T * 2 + (tok == 32 ? 1 : 0)) {
+    case 1 * 2: return max_pairs<1, 64>();
+    case 2 * 2: return max_pairs<2, 64>();
+    case 3 * 2: return max_pairs<3, 64>();
+    case 4 * 2: return max_pairs<4, 64>();
+    case 1 * 2 + 1: return max_pairs<1, 32>();
+    case 2 * 2 + 1: return max_pairs<2, 32>();
+    case 3 * 2 + 1: return max_pairs<3, 32>();
+    case 4 * 2 + 1: return max_pairs<4, 32>();
+  }
+  return 0;
 }
 
 }  // namespace pfl
@@ -507,7 +656,15 @@ namespace {
 std::mutex g_pfl_mu;
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 int g_pfl_sms[64];
+int g_pfl_pairs[64][4][2];   // [device][T - 1][tok == 32]: resident CTA pairs + 1 (0 = unknown)
 }  // namespace
+
+static int pfl_resident_pairs(int dev, int T, int tok) {
+  std::lock_guard<std::mutex> lock(g_pfl_mu);
+  int& v = g_pfl_pairs[dev][T - 1][tok == 32 ? 1 : 0];
+  if (v == 0) v = pfl::max_pairs_t(T, tok) + 1;
+  return v - 1;
+}
 
 static PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
   std::lock_guard<std::mutex> lock(g_pfl_mu);
@@ -586,7 +743,24 @@ fairy2i_status launch_wl_prefill_group(const void* x, fairy2i_dtype xdt, int64_t
   a.tok_tiles = (int)((B + tok - 1) / tok);
   const int64_t tiles = (int64_t)count * a.row_blocks * a.tok_tiles;
   if (tiles > (int64_t(1) << 30)) return FAIRY2I_OK;
-  const int grid = (int)(tiles < g_pfl_sms[dev] ? tiles : g_pfl_sms[dev]);
+  const int sms = g_pfl_sms[dev];
+  int grid = (int)(tiles < sms ? tiles : sms);
+  // K split over CTA pairs where it shortens the launch: in full-tile time, a pair finishes a
+  // tile in half the time, so ceil(tiles / pairs) / 2 waves against ceil(tiles / SMs); taken
+  // when that is at most 0.9 of it (the split adds a hand-over per tile) and every rank has a
+  // chunk.
+  a.split = 1;
+  if (a.nch >= 2) {
+    const int pairs = pfl_resident_pairs(dev, T, tok);
+    if (pairs > 0) {
+      const int64_t full_waves = (tiles + sms - 1) / sms;
+      const int64_t half_waves = (tiles + pairs - 1) / pairs;
+      if (half_waves * 5 <= full_waves * 9) {
+        a.split = 2;
+        grid = 2 * (int)(tiles < pairs ? tiles : pairs);
+      }
+    }
+  }
   *handled = true;
   switch (T * 2 + (tok == 32 ? 1 : 0)) {
     case 1 * 2: return launch<1, 64>(a, xre, xim, grid, stream);

@@ -276,8 +276,7 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
   constexpr int kPart = Lay::kPart;
   static_assert(NV <= kPart && NV <= 2 * kEpiThreads, "partial size");
   extern __shared__ unsigned char smem_raw[];
-  unsigned char* smem = reinterpret_cast<unsigned char*>(
-      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  unsigned char* smem = align_smem_1024(smem_raw);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kOffBar);
   uint64_t* full = bars;                        // [stage] codes landed        (tx count)
   uint64_t* empty = full + kMaxStages;          // [stage] codes read          (4 warps x nu)

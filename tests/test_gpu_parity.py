@@ -324,11 +324,14 @@ def test_retired_path_2_is_rejected(F):
     # 32-token tiles (B <= 32, two issuing threads per sign plane): full, ragged, the boundary
     (4096, 4096, 2, 16), (11008, 4096, 2, 32), (4096, 11008, 3, 31), (300, 1024, 4, 17),
     (64, 256, 1, 33), (2048, 2048, 2, 1),
+    # K split over CTA pairs (few tiles): 21 + 22 chunks, 2 + 3, 1 + 1, several tiles per pair
+    (4096, 11008, 2, 64), (100, 1280, 4, 40), (130, 400, 1, 129), (11008, 4096, 3, 20),
 ])
 def test_wl_tcgen05_prefill_path(F, out_f, in_f, T, B):
     """The tcgen05 prefill GEMM (path 3): ragged row blocks (R = 64, 32, 16, 16 rows of every
     stage-matrix for T = 1..4), ragged token tiles (32 tokens up to a batch of 32, else 64),
-    ragged 64-code x stages and 128-code chunks, one CTA or many tiles per CTA."""
+    ragged 64-code x stages and 128-code chunks, one CTA or many tiles per CTA, and the K split
+    over CTA pairs that launches of few tiles take."""
     n, m = O.complex_dims(out_f, in_f)
     codes, scales = _random_quantized(n, m, T, seed=5 * out_f + 3 * in_f + T)
     x = synth.outlier_activations(B, in_f, seed=out_f + in_f + 2)
@@ -431,6 +434,7 @@ def test_bounded_wait_latches_timeout_and_context_survives(F):
     (64, 256, 2, 5, 2, torch.bfloat16),       # 2 <= B <= 8: the chained kernel, 4 + 1 tokens
     (64, 256, 2, 12, 2, torch.bfloat16),      # B > 8: one prefill launch for the group
     (4096, 4096, 2, 64, 3, torch.bfloat16),   # the 7B q/k/v at 64 tokens: 192 tiles, one launch
+    (11008, 4096, 2, 64, 2, torch.bfloat16),  # gate / up at 64 tokens: K split, 4-5 tiles a pair
     (300, 512, 3, 130, 2, torch.bfloat16),    # ragged rows, three token tiles
     (37, 53, 2, 1, 4, torch.float32),         # fp32 x: members on the general path
 ])
