@@ -316,10 +316,10 @@ def run_ours(args, world, rank, local):
     calls, x_all, y_all = make_calls(linears, B, dev, groups)
     step_bytes = sum(call_bytes(c, B) for c in calls)
     nlinears = sum(len(c["members"]) for c in calls)
-    # a grouped call is one launch per token (B = 1) or per 4 tokens (2 <= B <= 8) where a decode
-    # kernel takes it, else one per member
-    launches_per_step = (len(calls) if B == 1 else len(calls) * ((B + 3) // 4) if B <= 8
-                         else nlinears)
+    # a grouped call is one launch: B = 1 on a decode kernel, 2 <= B <= 4 on the chained kernel,
+    # larger batches on the prefill GEMM; on the chained kernel chosen explicitly (path 5) one
+    # launch per 4 tokens
+    launches_per_step = (len(calls) * ((B + 3) // 4) if args.decode_path == 5 else len(calls))
 
     def step():
         for c in calls:
@@ -390,7 +390,7 @@ def run_ours(args, world, rank, local):
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
     traffic = decode_traffic(calls, args.decode_path, B, sms)
     kernels = (sorted({decode_kernel(c, args.decode_path, sms) for c in calls}) if B == 1 else
-               ["chain"] if B <= 8 and args.decode_path in (0, 5) else [])
+               ["chain"] if (B <= 4 and args.decode_path == 0) or args.decode_path == 5 else [])
     kname = ("wl_matmul decode (all launches of the step: "
              + " + ".join({"fp8": "warp-MMA", "stream": "persistent tcgen05",
                            "chain": "chained tcgen05"}[k] for k in kernels)
@@ -499,7 +499,7 @@ def run_batches(F, linears, dev, args):
         if name.startswith("mlp"):
             rec["us_per_layer"] = round(ms * 1e3 / len(linears), 2)
         rec["path"] = ("persistent tcgen05, one-token form" if B == 1 else
-                       "chained tcgen05, up to 4 tokens per launch" if B <= 8 else
+                       "chained tcgen05, one launch per call" if B <= 4 else
                        "tcgen05 GEMM (%d-token tiles; K split over CTA pairs where the "
                        "tiles fill the SMs poorly)" % (32 if B <= 32 else 64))
         out.append(rec)

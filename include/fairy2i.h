@@ -166,9 +166,10 @@ fairy2i_status fairy2i_wl_matmul(const void* x, fairy2i_dtype xdt, int64_t B,
 /* Same as fairy2i_wl_matmul with the kernel chosen by `path`:
  *   0 = automatic, every decode choice meeting the per-element bound for any x: B = 1 -> the
  *       persistent tcgen05 kernel's one-token form (4) for bf16 x, the chained kernel (5) for
- *       float32 x; 2 <= B <= 8 -> the chained kernel, up to 4 tokens per launch (skinny batch);
- *       (decode kernels: T <= 4, in_features <= 24576); B > 8 -> the tcgen05 prefill GEMM where
- *       it applies (see 3); otherwise the general CUDA-core kernel;
+ *       float32 x; 2 <= B <= 4 -> the chained kernel, one launch (skinny batch); (decode
+ *       kernels: T <= 4, in_features <= 24576); B > 4 -> the tcgen05 prefill GEMM where it
+ *       applies (see 3), else up to B = 8 the chained kernel (4 tokens per launch); otherwise
+ *       the general CUDA-core kernel;
  *   1 = the warp-MMA decode kernel (x as two e4m3 limbs, B <= 2) where it applies, otherwise
  *       the general kernel;
  *   2 = retired (an earlier tcgen05 decode kernel); returns FAIRY2I_ERR_INVALID_ARG;
@@ -220,10 +221,11 @@ fairy2i_status fairy2i_codes_adjoint(const uint32_t* codes, int64_t n, int64_t m
  * or the gate and up projections of a decoder layer: for g < count,
  *   y[g] = fairy2i_wl_matmul(x, xdt, B, in_features, ldx, codes[g], scales[g], out_features, T)
  * with codes[g], scales[g], y[g] device pointers passed in host arrays of `count` entries
- * (1 <= count <= FAIRY2I_MAX_GROUP). Where the automatic decode path applies (B <= 8, T <= 4,
- * in_features <= 24576) the whole group is one launch per token (B = 1: the persistent tcgen05
- * kernel's one-token form for bf16 x, the chained kernel for float32 x) or per 4 tokens (the
- * chained kernel); B > 8 bf16 tokens on the prefill GEMM: one launch holding every member's tiles;
+ * (1 <= count <= FAIRY2I_MAX_GROUP). Where the automatic decode path applies (B <= 4, T <= 4,
+ * in_features <= 24576) the whole group is one launch (B = 1: the persistent tcgen05 kernel's
+ * one-token form for bf16 x, the chained kernel for float32 x; 2 <= B <= 4: the chained
+ * kernel); B > 4 bf16 tokens on the prefill GEMM: one launch holding every member's tiles (up to
+ * B = 8 the chained kernel takes what the GEMM does not, 4 tokens per launch);
  * otherwise the members run one after the other on the automatic path. Requirements and errors are those of fairy2i_wl_matmul
  * for every member (checked before anything is enqueued); FAIRY2I_ERR_INVALID_ARG for a count
  * out of range or a null array. Results agree with the separate calls within the
@@ -238,6 +240,8 @@ fairy2i_status fairy2i_wl_matmul_group(const void* x, fairy2i_dtype xdt, int64_t
 
 /* fairy2i_wl_matmul_group with the decode kernel chosen by `path`: 0 = automatic (as above),
  * 1 = the warp-MMA decode kernel where it applies (else path 1 per member),
+ * 3 = the tcgen05 prefill GEMM, one launch for the group at any B (bf16 x with 16-byte aligned
+ * rows, m % 8 == 0, T <= 4; FAIRY2I_ERR_INVALID_ARG otherwise),
  * 4 = the persistent tcgen05 decode kernel, one launch for the group (B <= 2 bf16 tokens, T <= 4,
  * in_features <= 24576; FAIRY2I_ERR_INVALID_ARG for anything else), 5 = the chained decode kernel
  * on this one group (any B, up to 4 tokens per launch, T <= 4, in_features <= 24576;

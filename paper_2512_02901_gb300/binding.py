@@ -213,7 +213,8 @@ def wl_matmul_group(x: torch.Tensor, codes, scales, out_features: int, ys=None, 
                     T: int | None = None, path: int = PATH_AUTO):
     """Several linears of the same shape on one input x (CUDA): returns [y_g] with
     y_g = wl_matmul(x, codes[g], scales[g], out_features); one launch where a decode kernel
-    applies (path 0 automatic, 1 the warp-MMA decode kernel, 4 the persistent tcgen05 one)."""
+    applies (path 0 automatic, 1 the warp-MMA decode kernel, 3 the tcgen05 prefill GEMM at any B,
+    4 the persistent tcgen05 decode kernel, 5 the chained one)."""
     assert x.is_cuda and x.dim() == 2 and x.stride(1) == 1 and x.dtype in (torch.float32,
                                                                           torch.bfloat16)
     count = len(codes)

@@ -89,9 +89,13 @@ unsigned int* device_status_word() {
 
 static bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
-// Largest batch the automatic path sends to the chained kernel (skinny-batch decode); larger
-// batches take the tcgen05 prefill GEMM.
-constexpr int64_t kSkinnyMaxTokens = 8;
+// Largest batch the automatic path sends to the chained kernel first (skinny-batch decode: one
+// launch of up to 4 tokens per call); larger batches take the tcgen05 prefill GEMM, and the
+// chained kernel up to kChainMaxTokens what the GEMM does not take (float32 x, unaligned rows).
+// Measured per 7B layer (bf16, T = 2): the chained kernel 77-84 us at 2-4 tokens and 126-142 us
+// at 5-8 (two launches per call), the GEMM with K split ~112 us at 2-16.
+constexpr int64_t kSkinnyMaxTokens = 4;
+constexpr int64_t kChainMaxTokens = 8;
 
 // The automatic decode path (B <= 2 tokens): one token at a time through a kernel that holds
 // every x entry to the per-element bound for any x, i.e. to 2^-26 (persistent tcgen05 kernel,
@@ -266,6 +270,11 @@ fairy2i_status fairy2i_wl_matmul_path(const void* x, fairy2i_dtype xdt, int64_t 
     if (handled || st != FAIRY2I_OK) return st;
     if (path == 3) return FAIRY2I_ERR_INVALID_ARG;   // outside the prefill kernel's domain
   }
+  if (path == 0 && B > kSkinnyMaxTokens && B <= kChainMaxTokens) {   // not the GEMM's: chained
+    st = chain_tokens(x, xdt, B, in_features, ldx, 1, &codes, &scales, out_features, T, &y, ldy,
+                      s, &handled);
+    if (handled || st != FAIRY2I_OK) return st;
+  }
   if (path == 4) {   // persistent tcgen05 decode kernel (explicit): B <= 2 bf16 tokens, T <= 4
     st = launch_wl_stream_group(x, xdt, B, in_features, ldx, 1, &codes, &scales, n, m,
                                 out_features, wpr, T, &y, ldy, s, &handled);
@@ -308,7 +317,7 @@ fairy2i_status fairy2i_wl_matmul_group_path(const void* x, fairy2i_dtype xdt, in
                                             int T, float* const* y, int64_t ldy, int path,
                                             void* stream) {
   if (count < 1 || count > FAIRY2I_MAX_GROUP || !codes || !scales || !y ||
-      (path != 0 && path != 1 && path != 4 && path != 5))
+      (path != 0 && path != 1 && path != 3 && path != 4 && path != 5))
     return FAIRY2I_ERR_INVALID_ARG;
   // Every member is validated as a single call would be (B = 0 included) before anything runs.
   for (int g = 0; g < count; ++g) {
@@ -332,10 +341,16 @@ fairy2i_status fairy2i_wl_matmul_group_path(const void* x, fairy2i_dtype xdt, in
     if (handled || st != FAIRY2I_OK) return st;
     if (path == 5) return FAIRY2I_ERR_INVALID_ARG;
   }
-  if (B > kSkinnyMaxTokens && path == 0) {   // one prefill GEMM launch for the whole group
+  if (path == 3 || (B > kSkinnyMaxTokens && path == 0)) {   // one prefill GEMM launch
     const fairy2i_status st = launch_wl_prefill_group(x, xdt, B, in_features, ldx, count, codes,
                                                       scales, n, m, out_features, wpr, T, y, ldy,
                                                       s, &handled);
+    if (handled || st != FAIRY2I_OK) return st;
+    if (path == 3) return FAIRY2I_ERR_INVALID_ARG;   // outside the prefill kernel's domain
+  }
+  if (path == 0 && B > kSkinnyMaxTokens && B <= kChainMaxTokens) {   // not the GEMM's: chained
+    const fairy2i_status st = chain_tokens(x, xdt, B, in_features, ldx, count, codes, scales,
+                                           out_features, T, y, ldy, s, &handled);
     if (handled || st != FAIRY2I_OK) return st;
   }
   if (B <= 2 && path == 0) {   // per token, one launch for the whole group

@@ -122,11 +122,17 @@ def test_wl_matmul_group_validation(lib):
     assert call(ldx=15) == 2 and call(ldy=15) == 2
     assert call(codes=arr(GOOD, ODD, GOOD, GOOD)) == 3        # a misaligned member
     assert call(ys=arr(GOOD, GOOD, None, GOOD)) == 1          # a null member
-    # the group call with an explicit kernel: only paths 0, 1, 4 and 5 exist for a group
+    # the group call with an explicit kernel: only paths 0, 1, 3, 4 and 5 exist for a group
     cp = arr(*([GOOD] * 4))
-    for path in (2, 3, 6, -1):
+    for path in (2, 6, -1):
         assert lib.fairy2i_wl_matmul_group_path(GOOD, 1, 1, 16, 16, 3, cp, cp, 16, 2, cp, 16,
                                                 path, None) == 1
+    # path 3 (the prefill GEMM) outside its domain, rejected before any launch: float32 x, and
+    # m = 6 complex inputs (m % 8 != 0)
+    assert lib.fairy2i_wl_matmul_group_path(GOOD, 0, 1, 16, 16, 3, cp, cp, 16, 2, cp, 16, 3,
+                                            None) == 1
+    assert lib.fairy2i_wl_matmul_group_path(GOOD, 1, 1, 12, 16, 3, cp, cp, 16, 2, cp, 16, 3,
+                                            None) == 1
     assert lib.fairy2i_wl_matmul_group_path(GOOD, 1, 0, 16, 16, 3, cp, cp, 16, 2, cp, 16, 4,
                                             None) == 0     # empty batch on path 4
 

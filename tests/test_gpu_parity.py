@@ -378,7 +378,7 @@ def test_wl_tcgen05_prefill_strided_odd_input(F):
 
 
 def test_wl_auto_path_routes_batches_to_prefill(F):
-    """Above eight tokens the default path is the prefill GEMM where it applies: same bits."""
+    """Above four tokens the default path is the prefill GEMM where it applies: same bits."""
     n, m, T, B = 300, 512, 2, 33
     codes, scales = _random_quantized(n, m, T, seed=23)
     cd = upload_codes(O.pack_codes(codes))
@@ -426,13 +426,36 @@ def test_bounded_wait_latches_timeout_and_context_survives(F):
 
 
 # ------------------------------------------------------------------------------ grouped linears
+@pytest.mark.parametrize("out_f,in_f,T,B,count", [
+    (4096, 4096, 2, 5, 3),      # q/k/v shapes at 5 tokens: one K-split launch
+    (11008, 4096, 2, 8, 2),     # gate/up at 8 tokens
+    (300, 1024, 3, 3, 2),       # ragged rows, T = 3
+    (64, 256, 1, 2, 4),         # one 128-code chunk (no K split), four members
+])
+def test_group_prefill_path_any_batch(F, out_f, in_f, T, B, count):
+    """Path 3 for a group: one prefill GEMM launch holding every member's tiles, at skinny batches
+    too; every member matches the oracle."""
+    n, m = O.complex_dims(out_f, in_f)
+    layers = [_random_quantized(n, m, T, seed=61 + 5 * g + out_f) for g in range(count)]
+    x = synth.outlier_activations(B, in_f, seed=67 + in_f)
+    xd = x.to(DEV)
+    ys = F.wl_matmul_group(xd, [upload_codes(O.pack_codes(c)) for c, _ in layers],
+                           [torch.from_numpy(s).to(DEV) for _, s in layers], out_f, path=3)
+    assert F.get_status() == 0
+    xo = x.float().numpy()
+    for (c, s), yg in zip(layers, ys):
+        assert_wl_close(yg.cpu().numpy(), O.wl_matmul(xo, c, s, out_f), xo, s)
+
+
 @pytest.mark.parametrize("out_f,in_f,T,B,count,dtype", [
     (256, 512, 2, 1, 3, torch.bfloat16),      # one grouped decode launch (q, k, v shape class)
     (130, 258, 3, 2, 2, torch.bfloat16),      # ragged rows, two tokens
     (4096, 4096, 2, 1, 3, torch.bfloat16),    # the 7B attention projections
     (11008, 4096, 2, 1, 2, torch.bfloat16),   # the 7B gate and up projections
-    (64, 256, 2, 5, 2, torch.bfloat16),       # 2 <= B <= 8: the chained kernel, 4 + 1 tokens
-    (64, 256, 2, 12, 2, torch.bfloat16),      # B > 8: one prefill launch for the group
+    (64, 256, 2, 4, 2, torch.bfloat16),       # 2 <= B <= 4: the chained kernel, one launch
+    (64, 256, 2, 5, 2, torch.bfloat16),       # B > 4: one prefill launch for the group
+    (64, 254, 2, 6, 2, torch.float32),        # float32 x at 6 tokens: the chained kernel, 4 + 2
+    (64, 256, 2, 12, 2, torch.bfloat16),      # one prefill launch for the group
     (4096, 4096, 2, 64, 3, torch.bfloat16),   # the 7B q/k/v at 64 tokens: 192 tiles, one launch
     (11008, 4096, 2, 64, 2, torch.bfloat16),  # gate / up at 64 tokens: K split, 4-5 tiles a pair
     (300, 512, 3, 130, 2, torch.bfloat16),    # ragged rows, three token tiles

@@ -1,5 +1,6 @@
 """GPU parity of the skinny-batch decode (the chained kernel with 2 or 4 tokens per launch: the
-automatic path for 2 <= B <= 8, and wl_matmul path 5 for any B) against the CPU oracle: every
+automatic path for 2 <= B <= 4, and for 5 <= B <= 8 where the prefill GEMM does not apply, and
+wl_matmul path 5 for any B) against the CPU oracle: every
 token of ragged and full-size layers, T = 1..4, float32 and bf16 x, strided x and y, grouped
 linears, launches of 4, 2 and 1 tokens, an x of extreme range in every token. Tolerance as
 everywhere: relative Frobenius <= 1e-5 and |err| <= 1e-4 ||x~||_1 sum_t s_t per element."""
@@ -58,10 +59,11 @@ def _tokens(B, in_f, seed, dtype):
     (31, 515, 2, 3, torch.bfloat16, 0),       # ragged: launches of 2 + 1 tokens
     (64, 256, 3, 4, torch.float32, 0),
     (4096, 4096, 2, 4, torch.bfloat16, 0),    # the 7B attention projection, one launch of 4
-    (4096, 4096, 4, 5, torch.bfloat16, 0),    # T = 4: 4 + 1
-    (11008, 4096, 2, 8, torch.bfloat16, 0),   # gate / up: 4 + 4
-    (4096, 11008, 2, 6, torch.bfloat16, 0),   # down (43 chunks per row): 4 + 2
-    (100, 8192, 1, 7, torch.float32, 0),      # T = 1, long rows: 4 + 2 + 1
+    (4096, 4096, 4, 5, torch.bfloat16, 5),    # T = 4: 4 + 1
+    (11008, 4096, 2, 8, torch.bfloat16, 5),   # gate / up: 4 + 4
+    (4096, 11008, 2, 6, torch.bfloat16, 5),   # down (43 chunks per row): 4 + 2
+    (100, 8192, 1, 7, torch.float32, 0),      # T = 1, long rows, float32 x (automatic): 4 + 2 + 1
+    (64, 1000, 2, 6, torch.float32, 0),       # float32 x at 6 tokens (automatic): 4 + 2
     (130, 24576, 2, 4, torch.bfloat16, 5),    # the longest row the kernel takes
     (17, 2, 2, 2, torch.float32, 5),          # a single complex input
     (48, 1024, 3, 16, torch.bfloat16, 5),     # path 5 for any batch: four launches of 4
@@ -94,14 +96,14 @@ def test_skinny_strided_x_and_y(F):
     assert torch.all(yb[:, out_f:] == -7.0)
 
 
-@pytest.mark.parametrize("count,B", [(3, 4), (2, 3), (2, 8)])
-def test_skinny_group_matches_oracle(F, count, B):
+@pytest.mark.parametrize("count,B,path", [(3, 4, 0), (2, 3, 0), (2, 8, 5), (2, 6, 5)])
+def test_skinny_group_matches_oracle(F, count, B, path):
     out_f, in_f, T = 4096, 4096, 2
     n, m = O.complex_dims(out_f, in_f)
     layers = [_random_quantized(n, m, T, seed=40 + g) for g in range(count)]
     x = _tokens(B, in_f, seed=41, dtype=torch.bfloat16)
     ys = F.wl_matmul_group(x.to(DEV), [_upload(c) for c, _ in layers],
-                           [torch.from_numpy(s).to(DEV) for _, s in layers], out_f)
+                           [torch.from_numpy(s).to(DEV) for _, s in layers], out_f, path=path)
     assert F.get_status() == 0
     xo = x.float().numpy().astype(np.float64)
     for (c, s), yg in zip(layers, ys):

@@ -165,15 +165,16 @@ def test_stream_rejects_outside_its_domain(F):
 
 
 def test_automatic_decode_kernels(F):
-    """The automatic path runs one token (bf16 x) on the persistent kernel's one-token form and
-    2 to 8 tokens on the chained kernel (path 5), one launch for a whole group: bit for bit the
-    results of the explicit paths (every kernel is deterministic for a given launch shape)."""
+    """The automatic path runs one token (bf16 x) on the persistent kernel's one-token form, 2 to
+    4 tokens on the chained kernel (path 5) and 5 or more bf16 tokens on the prefill GEMM (path
+    3), one launch for a whole group: bit for bit the results of the explicit paths (every
+    kernel is deterministic for a given launch shape)."""
     out_f, in_f, T = 4096, 4096, 2
     n, m = O.complex_dims(out_f, in_f)
     layers = [_random_quantized(n, m, T, seed=81 + g) for g in range(3)]
     cds = [_upload(c) for c, _ in layers]
     scs = [torch.from_numpy(s).to(DEV) for _, s in layers]
-    for B, path in ((1, PATH), (2, 5), (5, 5)):
+    for B, path in ((1, PATH), (2, 5), (4, 5), (5, 3), (8, 3)):
         x = synth.outlier_activations(B, in_f, seed=83 + B).to(DEV)
         auto_group = F.wl_matmul_group(x, cds, scs, out_f)
         explicit = F.wl_matmul_group(x, cds, scs, out_f, path=path)
