@@ -74,9 +74,9 @@ DECODE_DRAM_BYTES = {
             "q": 4.231e6, "k": 4.231e6, "v": 4.231e6, "gate": 11.309e6, "up": 11.309e6},
     "stream": {"q,k,v": 12.655e6, "o": 4.265e6, "gate,up": 22.616e6, "down": 11.357e6},
 }
-PREFILL_T2_UP_DRAM_BYTES = 28.089e6 + 36.948e6
+PREFILL_T2_UP_DRAM_BYTES = 28.105e6 + 37.335e6
 # ncu sm__pipe_tensor_cycles_active of the same prefill launch (T = 2, up layer, 2048 tokens)
-PREFILL_T2_UP_TENSOR_PIPE_PCT = 52.7
+PREFILL_T2_UP_TENSOR_PIPE_PCT = 52.8
 
 
 def decode_kernel(c, path, sms):
