@@ -216,6 +216,12 @@ __device__ __forceinline__ uint32_t cluster_ctarank() {
 __device__ __forceinline__ void cluster_arrive() {
   asm volatile("barrier.cluster.arrive.release;" ::: "memory");
 }
+// The arrive without memory ordering, for a first phase whose only purpose is that every rank's
+// mbarriers are initialised before a peer uses them: the initialising thread publishes them with
+// fence.mbarrier_init.release.cluster, and the wait (acquire) pairs with that fence.
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed;" ::: "memory");
+}
 __device__ __forceinline__ void cluster_wait() {
   asm volatile("barrier.cluster.wait.acquire;" ::: "memory");
 }

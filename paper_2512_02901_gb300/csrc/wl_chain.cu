@@ -394,7 +394,7 @@ __global__ void __launch_bounds__(kThreads, 1) wl_chain_kernel(const __grid_cons
     __syncwarp();
     if (lane == 0) mbar_arrive(sfready);
   }
-  if (ks > 1) cluster_arrive();   // barriers of every rank initialised (waited before DSMEM use)
+  if (ks > 1) cluster_arrive_relaxed();   // every rank's barriers initialised (waited before DSMEM use)
   pdl_launch_dependents();
 
   if (warp < kDecWarps) {

@@ -239,7 +239,7 @@ __global__ void __launch_bounds__(Cfg<TOK>::kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  if (split) cluster_arrive();   // both ranks' barriers initialised (waited before remote use)
+  if (split) cluster_arrive_relaxed();   // both ranks' barriers initialised (waited before remote use)
   pdl_launch_dependents();
 
   if (warp == kCopyWarp) {
