@@ -471,9 +471,10 @@ __global__ void __launch_bounds__(Layout<NB>::kThreads, 1) wl_stream_kernel(cons
     const int ii = warp - kIssWarp0, set = ii / kIss, e = ii % kIss;
     if (lane == 0) {
       const uint32_t b_base = smem_u32(smem + kOffB);
+      // the scale factors are stored long before the B tiles: waited off the critical path
+      bool ok = !kF4 || wait_or_abort(sfready, 0, abort_flag, a.status);
       pdl_wait_primary();   // the B tiles are built from x after the previous kernel
-      bool ok = wait_or_abort(bready, 0, abort_flag, a.status);
-      if (kF4 && ok) ok = wait_or_abort(sfready, 0, abort_flag, a.status);
+      if (ok) ok = wait_or_abort(bready, 0, abort_flag, a.status);
       tc_fence_after();
       bool issued = false;
       int cur = -1;
