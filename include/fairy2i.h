@@ -188,10 +188,11 @@ fairy2i_status fairy2i_wl_matmul(const void* x, fairy2i_dtype xdt, int64_t B,
  *       per launch (the decoded signs feed the MMAs of every token of the launch); it takes any
  *       B (float32 or bf16 x), T <= 4 and in_features <= 24576 and returns
  *       FAIRY2I_ERR_INVALID_ARG for anything else.
- * The decode kernels (paths 1, 4) read the codes and scales before waiting for the previous
- * kernel in the stream (programmatic dependent launch): the codes must not be written by the
- * kernel launched right before the matmul on the same stream unless that kernel is one of this
- * library's convert/quantize/adjoint kernels, which end before any dependent kernel starts.
+ * The tensor-core kernels (paths 1, 3, 4, 5, and so the automatic path) read codes (the decode
+ * kernels also the scales) before waiting for the previous kernel in the stream (programmatic
+ * dependent launch): the codes must not be written by the kernel launched right before the
+ * matmul on the same stream unless that kernel is one of this library's convert/quantize/adjoint
+ * kernels, which end before any dependent kernel starts.
  * Results agree within the float32-accumulation tolerance whichever path runs. */
 fairy2i_status fairy2i_wl_matmul_path(const void* x, fairy2i_dtype xdt, int64_t B,
                                       int64_t in_features, int64_t ldx, const uint32_t* codes,

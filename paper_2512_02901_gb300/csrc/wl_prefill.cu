@@ -248,7 +248,9 @@ __global__ void __launch_bounds__(Cfg<TOK>::kThreads, 1)
       prefetch_tensormap(&xre);
       prefetch_tensormap(&xim);
     }
-    pdl_wait_primary();   // x may be written by the previous kernel
+    // The first code stage is copied before griddepcontrol.wait (codes are not written by a
+    // kernel that lets this one start early); x, which may be, after it.
+    bool waited = false;
     int xq = 0, cq = 0;   // running stage counters over all tiles of this CTA
     for (int it = 0; it < my_tiles && !__shfl_sync(0xffffffffu, *abort_flag, 0); ++it) {
       const int tile = unit + it * nunits;
@@ -280,6 +282,10 @@ __global__ void __launch_bounds__(Cfg<TOK>::kThreads, 1)
         if (lane == 0 && xq >= kXS)
           okx = wait_or_abort(&xempty[xst], ((xq / kXS) - 1) & 1, abort_flag, a.status);
         if (!__shfl_sync(0xffffffffu, okx, 0)) break;
+        if (!waited) {
+          pdl_wait_primary();
+          waited = true;
+        }
         if (lane == 0) {
           mbar_arrive_expect_tx(&xfull[xst], (uint32_t)kXStage);
           unsigned char* dst = smem + kOffX + xst * kXStage;
