@@ -23,13 +23,16 @@
 // are stored and x has landed) and one commit (plus one per x stage): the issue cost per MMA is
 // what bounds this kernel once the waits are per MMA.
 //
-// Roles (15 warps; warp w reaches TMEM lanes 32 (w % 4) ..): warps 0-7, two sets of four, decode
-// the code words into the A ring, set s taking pair s of every group (one 32-column store: sigma,
-// tau of two steps, left in flight while the next group is decoded), warp 0 also relaying the
-// x-stage arrival into the group barrier; they run on into the next tile without a pause. Warps
-// 8 and 9 issue the sigma and the tau MMAs; warp 10 copies the codes (bulk copies of whole 16-row
-// tiles) and x (TMA) in; warps 11-14 run the epilogue of each tile (every accumulator column is
-// read out first, so the MMAs of the next tile start before the reduction and the stores).
+// Roles (16 warps, 18 at 32-token tiles; warp w reaches TMEM lanes 32 (w % 4) ..): warps 0-7,
+// two sets of four, decode the code words into the A ring, set s taking pair s of every group
+// (one 32-column store: sigma, tau of two steps, left in flight while the next group is decoded),
+// warp 0 also relaying the x-stage arrival into the group barrier; they run on into the next
+// tile without a pause. Warps
+// 8 and 9 issue the sigma and the tau MMAs (8-11 at 32-token tiles); the next warp copies x in
+// (TMA) and the one after it the codes (bulk copies of whole 16-row tiles), each on its own since
+// a thread blocks for a while on every copy it issues; the last four run the epilogue of each tile
+// (every accumulator column is read out first, so the MMAs of the next tile start before the
+// reduction and the stores).
 //
 // K split over CTA pairs. When the tiles fill the SMs poorly (a few tiles per SM, as at batches of
 // up to 64 tokens: 64 tiles of an attention output projection on 152 SMs) the launch is made of
@@ -74,8 +77,9 @@ template <int TOK>
 struct Cfg {
   static constexpr int kIssPP = TOK == 32 ? 2 : 1;          // issuing threads per sign plane
   static constexpr int kIssN = 2 * kIssPP;
-  static constexpr int kCopyWarp = kIssWarp + kIssN;
-  static constexpr int kEpiWarp = kCopyWarp + 1;            // 4 epilogue warps
+  static constexpr int kCopyWarp = kIssWarp + kIssN;        // x (TMA)
+  static constexpr int kCodeWarp = kCopyWarp + 1;           // codes (bulk copies)
+  static constexpr int kEpiWarp = kCodeWarp + 1;            // 4 epilogue warps
   static constexpr int kThreads = (kEpiWarp + 4) * 32;
   static constexpr int kN = 2 * TOK;                        // B rows: Re x, then Im x
   static constexpr int kAccCols = kN;                       // columns of one accumulator
@@ -243,46 +247,28 @@ __global__ void __launch_bounds__(Cfg<TOK>::kThreads, 1)
   pdl_launch_dependents();
 
   if (warp == kCopyWarp) {
-    // ---------------- producer: codes (bulk copies) and x (TMA), in K order ----------------
+    // ---------------- producer of x (TMA), in K order ----------------
     if (lane == 0) {
       prefetch_tensormap(&xre);
       prefetch_tensormap(&xim);
     }
-    // The first code stage is copied before griddepcontrol.wait (codes are not written by a
-    // kernel that lets this one start early); x, which may be, after it.
     bool waited = false;
-    int xq = 0, cq = 0;   // running stage counters over all tiles of this CTA
+    int xq = 0;   // running stage counter over all tiles of this CTA
     for (int it = 0; it < my_tiles && !__shfl_sync(0xffffffffu, *abort_flag, 0); ++it) {
       const int tile = unit + it * nunits;
       int g, rb, tb;
       tile_coords(a, tile, g, rb, tb);
-      const uint32_t* codes = a.codes[g];
-      int ntl = 0;
-#pragma unroll
-      for (int rt = 0; rt < RT; ++rt) ntl += (rb * RT + rt < a.row_tiles) ? 1 : 0;
+      bool ok = true;
       for (int xs = c0; xs < c0 + nch; ++xs, ++xq) {
-        if ((xs - c0) % kCChunks == 0) {   // code stage: chunks xs .. xs + kCChunks - 1
-          const int st = cq % kCS;
-          const int nc = min(kCChunks, c0 + nch - xs);
-          bool ok = cq < kCS ||
-                    lane != 0 || wait_or_abort(&cempty[st], ((cq / kCS) - 1) & 1, abort_flag, a.status);
-          if (!__all_sync(0xffffffffu, ok)) break;
-          if (lane == 0) mbar_arrive_expect_tx(&cfull[st], (uint32_t)(TM * ntl * nc * 512));
-          __syncwarp();
-          const int tm = lane / RT, rt = lane % RT;
-          if (lane < TM * RT && rt < ntl) {
-            const int64_t t16 = (int64_t)tm * a.row_tiles + rb * RT + rt;
-            bulk_load(smem + kOffCodes + st * kCStage + lane * kCChunks * 512,
-                      codes + (t16 * a.nch + xs) * 128, (uint32_t)(nc * 512), &cfull[st]);
-          }
-          ++cq;
-        }
         const int xst = xq % kXS;
         bool okx = true;
         if (lane == 0 && xq >= kXS)
           okx = wait_or_abort(&xempty[xst], ((xq / kXS) - 1) & 1, abort_flag, a.status);
-        if (!__shfl_sync(0xffffffffu, okx, 0)) break;
-        if (!waited) {
+        if (!__shfl_sync(0xffffffffu, okx, 0)) {
+          ok = false;
+          break;
+        }
+        if (!waited) {   // x may be written by the previous kernel
           pdl_wait_primary();
           waited = true;
         }
@@ -296,15 +282,51 @@ __global__ void __launch_bounds__(Cfg<TOK>::kThreads, 1)
         }
         __syncwarp();
       }
+      if (!ok) break;
     }
     // Copies still in flight (after an abort) land before the CTA exits: wait for the last phase
     // of every stage that was filled.
-    if (lane == 0) {
+    if (lane == 0)
       for (int q = max(0, xq - kXS); q < xq; ++q)
         (void)mbar_wait_timed(&xfull[q % kXS], (q / kXS) & 1, kWaitNs);
+    __syncwarp();
+  } else if (warp == C::kCodeWarp) {
+    // ---- producer of the codes (bulk copies of whole 16-row tiles, kCChunks chunks a stage):
+    // its own warp, since a thread issuing copies blocks on each, and ahead of x (codes are not
+    // written by a kernel that lets this one start early, so no griddepcontrol.wait) ----
+    int cq = 0;   // running stage counter over all tiles of this CTA
+    for (int it = 0; it < my_tiles && !__shfl_sync(0xffffffffu, *abort_flag, 0); ++it) {
+      const int tile = unit + it * nunits;
+      int g, rb, tb;
+      tile_coords(a, tile, g, rb, tb);
+      const uint32_t* codes = a.codes[g];
+      int ntl = 0;
+#pragma unroll
+      for (int rt = 0; rt < RT; ++rt) ntl += (rb * RT + rt < a.row_tiles) ? 1 : 0;
+      bool ok = true;
+      for (int xs = c0; xs < c0 + nch; xs += kCChunks, ++cq) {   // chunks xs .. xs + nc - 1
+        const int st = cq % kCS;
+        const int nc = min(kCChunks, c0 + nch - xs);
+        ok = cq < kCS ||
+             lane != 0 || wait_or_abort(&cempty[st], ((cq / kCS) - 1) & 1, abort_flag, a.status);
+        if (!__all_sync(0xffffffffu, ok)) {
+          ok = false;
+          break;
+        }
+        if (lane == 0) mbar_arrive_expect_tx(&cfull[st], (uint32_t)(TM * ntl * nc * 512));
+        __syncwarp();
+        const int tm = lane / RT, rt = lane % RT;
+        if (lane < TM * RT && rt < ntl) {
+          const int64_t t16 = (int64_t)tm * a.row_tiles + rb * RT + rt;
+          bulk_load(smem + kOffCodes + st * kCStage + lane * kCChunks * 512,
+                    codes + (t16 * a.nch + xs) * 128, (uint32_t)(nc * 512), &cfull[st]);
+        }
+      }
+      if (!ok) break;
+    }
+    if (lane == 0)
       for (int q = max(0, cq - kCS); q < cq; ++q)
         (void)mbar_wait_timed(&cfull[q % kCS], (q / kCS) & 1, kWaitNs);
-    }
     __syncwarp();
   } else if (warp >= kIssWarp && warp < kIssWarp + kIssN) {
     // ---- MMA issuers: warp kIssWarp + kIssPP p + e issues, for sign plane p (sigma, tau), the
@@ -349,25 +371,34 @@ __global__ void __launch_bounds__(Cfg<TOK>::kThreads, 1)
     const int set = warp >> 2, quarter = warp & 3, L = quarter * 32 + lane;
     const uint32_t t_lane = tmem + ((uint32_t)(quarter * 32) << 16);
     const int tl = L >> 4, rl = L & 15;   // 16-row tile (tm * RT + rt) and row within it
-    const bool relay = warp == 0;         // waits for each x stage before arriving on its groups
+    const bool relay = warp == 0;         // waits for each x stage before announcing its groups
     int g = 0;                            // running group counter
     int cq0 = 0;                          // code stages of the earlier tiles
     for (int it = 0; it < my_tiles; ++it) {
       bool ok = true;
       // Software pipeline of one group: the A store of group g is in flight while group g + 1 is
-      // decoded; its barrier arrival follows the store wait at the next iteration.
-      int pend = -1;                      // slot of the group stored but not yet announced
+      // decoded; its barrier arrival follows the store wait at the next iteration (the relay
+      // warp's after the group's x stage has landed: only the MMAs need x, not the decode).
+      int pend = -1, pend_gi = 0;         // slot and group of the group stored, not announced
+      auto announce = [&]() -> bool {
+        tmem_wait_st();
+        tc_fence_before();
+        if (relay && (pend_gi & 1) == 0) {   // the first group of an x stage
+          const int xq = it * nch + (pend_gi >> 1);
+          bool okx = true;
+          if (lane == 0) okx = wait_or_abort(&xfull[xq % kXS], (xq / kXS) & 1, abort_flag, a.status);
+          if (!__shfl_sync(0xffffffffu, okx, 0)) return false;
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&gfull[pend]);
+        pend = -1;
+        return true;
+      };
       for (int gi = 0; gi < gpt; ++gi, ++g) {
         const int slot = g % kG;
         const int cq = cq0 + gi / kGroupsPerCStage, st = cq % kCS;
         if (gi % kGroupsPerCStage == 0)
           ok = __all_sync(0xffffffffu, wait_or_abort(&cfull[st], (cq / kCS) & 1, abort_flag, a.status));
-        if (ok && relay && (gi & 1) == 0) {   // x of this group landed (announced with the group)
-          const int xq = it * nch + (gi >> 1);
-          bool okx = true;
-          if (lane == 0) okx = wait_or_abort(&xfull[xq % kXS], (xq / kXS) & 1, abort_flag, a.status);
-          ok = __shfl_sync(0xffffffffu, okx, 0);
-        }
         if (!ok) break;
         const int wi = (gi % kGroupsPerCStage) * 4 + set * 2;   // first word of the pair in the stage
         const uint2 w2 = *reinterpret_cast<const uint2*>(
@@ -381,12 +412,9 @@ __global__ void __launch_bounds__(Cfg<TOK>::kThreads, 1)
         __syncwarp();
         if (lane == 0 && (gi % kGroupsPerCStage == kGroupsPerCStage - 1 || gi == gpt - 1))
           mbar_arrive(&cempty[st]);   // this warp's last read of the code stage
-        if (pend >= 0) {
-          tmem_wait_st();
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&gfull[pend]);
-          pend = -1;
+        if (pend >= 0 && !announce()) {
+          ok = false;
+          break;
         }
         if (g >= kG)
           ok = __all_sync(0xffffffffu, wait_or_abort(&gempty[slot], ((g / kG) - 1) & 1,
@@ -394,13 +422,9 @@ __global__ void __launch_bounds__(Cfg<TOK>::kThreads, 1)
         if (!ok) break;
         tmem_st32(t_lane + kColA + slot * 64 + set * 32, r);
         pend = slot;
+        pend_gi = gi;
       }
-      if (ok && pend >= 0) {
-        tmem_wait_st();
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&gfull[pend]);
-      }
+      if (ok && pend >= 0 && !announce()) ok = false;
       cq0 += (gpt + kGroupsPerCStage - 1) / kGroupsPerCStage;
       if (!ok) break;
     }
