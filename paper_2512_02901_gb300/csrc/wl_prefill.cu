@@ -18,10 +18,10 @@
 // share x in L2.
 //
 // Pipeline granularity: a group = 64 codes = 4 steps of 16 codes = 2 step pairs. The A ring holds
-// 4 groups (64 TMEM columns each); an x stage holds 128 codes (two groups). Per group an issuer
-// makes one barrier wait (the group's full barrier, which the decoders complete once the A pairs
-// are stored and x has landed) and one commit (plus one per x stage): the issue cost per MMA is
-// what bounds this kernel once the waits are per MMA.
+// 4 groups (64 TMEM columns each); an x stage holds 128 codes (two groups), which the decoders
+// take per iteration. Per group an issuer makes one barrier wait (the group's full barrier, which
+// the decoders complete once the A pairs are stored and x has landed) and one commit (plus one
+// per x stage): the issue cost per MMA is what bounds this kernel once the waits are per MMA.
 //
 // Roles (16 warps, 18 at 32-token tiles; warp w reaches TMEM lanes 32 (w % 4) ..): warps 0-7,
 // two sets of four, decode the code words into the A ring, set s taking pair s of every group
@@ -376,53 +376,68 @@ __global__ void __launch_bounds__(Cfg<TOK>::kThreads, 1)
     int cq0 = 0;                          // code stages of the earlier tiles
     for (int it = 0; it < my_tiles; ++it) {
       bool ok = true;
-      // Software pipeline of one group: the A store of group g is in flight while group g + 1 is
-      // decoded; its barrier arrival follows the store wait at the next iteration (the relay
-      // warp's after the group's x stage has landed: only the MMAs need x, not the decode).
-      int pend = -1, pend_gi = 0;         // slot and group of the group stored, not announced
+      // Two groups (the two halves of one x stage) per iteration, so that the waits and the
+      // barrier traffic are paid once per pair. Software pipeline: the A stores of a pair are in
+      // flight while the next pair is decoded; their barrier arrivals follow the store wait at the
+      // next iteration (the relay warp's after the pair's x stage has landed: only the MMAs need
+      // x, not the decode).
+      int pend = -1, pend_xq = 0;         // first slot and x stage of the pair stored, not announced
       auto announce = [&]() -> bool {
         tmem_wait_st();
         tc_fence_before();
-        if (relay && (pend_gi & 1) == 0) {   // the first group of an x stage
-          const int xq = it * nch + (pend_gi >> 1);
+        if (relay) {
           bool okx = true;
-          if (lane == 0) okx = wait_or_abort(&xfull[xq % kXS], (xq / kXS) & 1, abort_flag, a.status);
+          if (lane == 0)
+            okx = wait_or_abort(&xfull[pend_xq % kXS], (pend_xq / kXS) & 1, abort_flag, a.status);
           if (!__shfl_sync(0xffffffffu, okx, 0)) return false;
         }
         __syncwarp();
-        if (lane == 0) mbar_arrive(&gfull[pend]);
+        if (lane == 0) {
+          mbar_arrive(&gfull[pend]);
+          mbar_arrive(&gfull[pend + 1]);
+        }
         pend = -1;
         return true;
       };
-      for (int gi = 0; gi < gpt; ++gi, ++g) {
+      for (int gi = 0; gi < gpt; gi += 2, g += 2) {   // gpt, g even: slots g % kG, g % kG + 1
         const int slot = g % kG;
         const int cq = cq0 + gi / kGroupsPerCStage, st = cq % kCS;
         if (gi % kGroupsPerCStage == 0)
           ok = __all_sync(0xffffffffu, wait_or_abort(&cfull[st], (cq / kCS) & 1, abort_flag, a.status));
         if (!ok) break;
-        const int wi = (gi % kGroupsPerCStage) * 4 + set * 2;   // first word of the pair in the stage
-        const uint2 w2 = *reinterpret_cast<const uint2*>(
-            smem + kOffCodes + st * kCStage + (tl * kCChunks + (wi >> 3)) * 512 + rl * 32 +
-            (wi & 7) * 4);
+        // first word of pair `set` of group gi in the stage; group gi + 1's is 4 words on, in the
+        // same 128-code chunk
+        const int wi = (gi % kGroupsPerCStage) * 4 + set * 2;
+        const unsigned char* cw = smem + kOffCodes + st * kCStage +
+                                  (tl * kCChunks + (wi >> 3)) * 512 + rl * 32 + (wi & 7) * 4;
+        const uint2 w2a = *reinterpret_cast<const uint2*>(cw);
+        const uint2 w2b = *reinterpret_cast<const uint2*>(cw + 16);
         uint32_t r[32];
-        plane_bf16(prmt(w2.x, 0u, 0x1404u), r);        // sigma, first step of the pair
-        plane_bf16(prmt(w2.x, 0u, 0x3424u), r + 8);    // tau
-        plane_bf16(prmt(w2.y, 0u, 0x1404u), r + 16);   // sigma, second step
-        plane_bf16(prmt(w2.y, 0u, 0x3424u), r + 24);   // tau
-        __syncwarp();
-        if (lane == 0 && (gi % kGroupsPerCStage == kGroupsPerCStage - 1 || gi == gpt - 1))
-          mbar_arrive(&cempty[st]);   // this warp's last read of the code stage
+        plane_bf16(prmt(w2a.x, 0u, 0x1404u), r);        // sigma, first step of the pair
+        plane_bf16(prmt(w2a.x, 0u, 0x3424u), r + 8);    // tau
+        plane_bf16(prmt(w2a.y, 0u, 0x1404u), r + 16);   // sigma, second step
+        plane_bf16(prmt(w2a.y, 0u, 0x3424u), r + 24);   // tau
         if (pend >= 0 && !announce()) {
           ok = false;
           break;
         }
         if (g >= kG)
           ok = __all_sync(0xffffffffu, wait_or_abort(&gempty[slot], ((g / kG) - 1) & 1,
-                                                     abort_flag, a.status));
+                                                     abort_flag, a.status) &&
+                                           wait_or_abort(&gempty[slot + 1], ((g / kG) - 1) & 1,
+                                                         abort_flag, a.status));
         if (!ok) break;
         tmem_st32(t_lane + kColA + slot * 64 + set * 32, r);
+        plane_bf16(prmt(w2b.x, 0u, 0x1404u), r);
+        plane_bf16(prmt(w2b.x, 0u, 0x3424u), r + 8);
+        plane_bf16(prmt(w2b.y, 0u, 0x1404u), r + 16);
+        plane_bf16(prmt(w2b.y, 0u, 0x3424u), r + 24);
+        tmem_st32(t_lane + kColA + (slot + 1) * 64 + set * 32, r);
+        __syncwarp();
+        if (lane == 0 && ((gi + 1) % kGroupsPerCStage == kGroupsPerCStage - 1 || gi + 1 == gpt - 1))
+          mbar_arrive(&cempty[st]);   // this warp's last read of the code stage
         pend = slot;
-        pend_gi = gi;
+        pend_xq = it * nch + (gi >> 1);
       }
       if (ok && pend >= 0 && !announce()) ok = false;
       cq0 += (gpt + kGroupsPerCStage - 1) / kGroupsPerCStage;
