@@ -326,6 +326,7 @@ def test_retired_path_2_is_rejected(F):
     (64, 256, 1, 33), (2048, 2048, 2, 1),
     # K split over CTA pairs (few tiles): 21 + 22 chunks, 2 + 3, 1 + 1, several tiles per pair
     (4096, 11008, 2, 64), (100, 1280, 4, 40), (130, 400, 1, 129), (11008, 4096, 3, 20),
+    (1000, 2048, 1, 20), (4096, 4096, 1, 64), (200, 3008, 2, 7),
 ])
 def test_wl_tcgen05_prefill_path(F, out_f, in_f, T, B):
     """The tcgen05 prefill GEMM (path 3): ragged row blocks (R = 64, 32, 16, 16 rows of every
