@@ -102,6 +102,7 @@ struct Cfg {
 };
 
 constexpr int kMaxGroup = 4;
+constexpr int64_t kTwoLaunchMinTokens = 512;   // T = 3 as a T = 2 and a T = 1 launch from here on
 
 struct Args {
   const uint32_t* codes[kMaxGroup];   // linears sharing x (a group), same shape
@@ -116,6 +117,7 @@ struct Args {
   int row_blocks;   // ceil(n / R) per linear
   int tok_tiles;    // ceil(B / TOK)
   int split;        // 2: clusters of two CTAs split each tile's chunks; 1: one CTA per tile
+  int accumulate;   // 1: y += the result (the second launch of a two-launch T = 3 layer)
 };
 
 // Tile t (token-tile-major, so that CTAs (or CTA pairs) running together share x in L2): token
@@ -601,12 +603,19 @@ __global__ void __launch_bounds__(Cfg<TOK>::kThreads, 1)
           if (db < nb) {
             float* const yp = yt + db * a.ldy;
             if (vec) {
+              if (a.accumulate) {   // y (the first launch's stages) + this launch's, in that order
+                const float4 y0 = *reinterpret_cast<const float4*>(yp);
+                out.x = y0.x + out.x;
+                out.y = y0.y + out.y;
+                out.z = y0.z + out.z;
+                out.w = y0.w + out.w;
+              }
               *reinterpret_cast<float4*>(yp) = out;
             } else {
-              if (j < lim) yp[0] = out.x;
-              if (j + 1 < lim) yp[1] = out.y;
-              if (j + 2 < lim) yp[2] = out.z;
-              if (j + 3 < lim) yp[3] = out.w;
+              const float v[4] = {out.x, out.y, out.z, out.w};
+#pragma unroll
+              for (int c = 0; c < 4; ++c)
+                if (j + c < lim) yp[c] = a.accumulate ? yp[c] + v[c] : v[c];
             }
           }
         }
@@ -772,53 +781,70 @@ fairy2i_status launch_wl_prefill_group(const void* x, fairy2i_dtype xdt, int64_t
   const bool has_im = in_features > m;
   if (!encode_x_map(&xim, has_im ? xb + m : xb, has_im ? in_features - m : 1, B, ldx, tok))
     return FAIRY2I_OK;
-  const int R = T == 1 ? 64 : (T == 2 ? 32 : 16);
-  Args a;
-  for (int g = 0; g < kMaxGroup; ++g) {
-    const int gg = g < count ? g : 0;
-    a.codes[g] = codes[gg];
-    a.scales[g] = scales[gg];
-    a.y[g] = y[gg];
-  }
-  a.G = count;
-  a.status = device_status_word();
-  a.B = B; a.n = n; a.out_features = out_features; a.ldy = ldy;
-  a.wpr = (int)wpr; a.nch = (int)(wpr / 8); a.row_tiles = (int)((n + 15) / 16);
-  a.row_blocks = (int)((n + R - 1) / R);
-  a.tok_tiles = (int)((B + tok - 1) / tok);
-  const int64_t tiles = (int64_t)count * a.row_blocks * a.tok_tiles;
-  if (tiles > (int64_t(1) << 30)) return FAIRY2I_OK;
-  const int sms = g_pfl_sms[dev];
-  int grid = (int)(tiles < sms ? tiles : sms);
-  // K split over CTA pairs where it shortens the launch: in full-tile time, a pair finishes a
-  // tile in half the time, so ceil(tiles / pairs) / 2 waves against ceil(tiles / SMs); taken
-  // when that is at most 0.9 of it (the split adds a hand-over per tile) and every rank has a
-  // chunk.
-  a.split = 1;
-  if (a.nch >= 2) {
-    const int pairs = pfl_resident_pairs(dev, T, tok);
-    if (pairs > 0) {
-      const int64_t full_waves = (tiles + sms - 1) / sms;
-      const int64_t half_waves = (tiles + pairs - 1) / pairs;
-      if (half_waves * 5 <= full_waves * 9) {
-        a.split = 2;
-        grid = 2 * (int)(tiles < pairs ? tiles : pairs);
+  // One launch over stages [t0, t0 + Tp) of every member; accumulate: y += its result.
+  auto run = [&](int Tp, int t0, int accumulate) -> fairy2i_status {
+    const int R = Tp == 1 ? 64 : (Tp == 2 ? 32 : 16);
+    // words of one stage-matrix's codes ([T][2][row tile][chunk][16 rows][8 words] per member)
+    const int64_t sm_words = ((n + 15) / 16) * 16 * wpr;
+    Args a;
+    for (int g = 0; g < kMaxGroup; ++g) {
+      const int gg = g < count ? g : 0;
+      a.codes[g] = codes[gg] + (int64_t)t0 * 2 * sm_words;
+      a.scales[g] = scales[gg] + t0 * 4;
+      a.y[g] = y[gg];
+    }
+    a.G = count;
+    a.accumulate = accumulate;
+    a.status = device_status_word();
+    a.B = B; a.n = n; a.out_features = out_features; a.ldy = ldy;
+    a.wpr = (int)wpr; a.nch = (int)(wpr / 8); a.row_tiles = (int)((n + 15) / 16);
+    a.row_blocks = (int)((n + R - 1) / R);
+    a.tok_tiles = (int)((B + tok - 1) / tok);
+    const int64_t tiles = (int64_t)count * a.row_blocks * a.tok_tiles;
+    const int sms = g_pfl_sms[dev];
+    int grid = (int)(tiles < sms ? tiles : sms);
+    // K split over CTA pairs where it shortens the launch: in full-tile time, a pair finishes a
+    // tile in half the time, so ceil(tiles / pairs) / 2 waves against ceil(tiles / SMs); taken
+    // when that is at most 0.9 of it (the split adds a hand-over per tile) and every rank has a
+    // chunk.
+    a.split = 1;
+    if (a.nch >= 2) {
+      const int pairs = pfl_resident_pairs(dev, Tp, tok);
+      if (pairs > 0) {
+        const int64_t full_waves = (tiles + sms - 1) / sms;
+        const int64_t half_waves = (tiles + pairs - 1) / pairs;
+        if (half_waves * 5 <= full_waves * 9) {
+          a.split = 2;
+          grid = 2 * (int)(tiles < pairs ? tiles : pairs);
+        }
       }
     }
+    switch (Tp * 2 + (tok == 32 ? 1 : 0)) {
+      case 1 * 2: return launch<1, 64>(a, xre, xim, grid, stream);
+      case 2 * 2: return launch<2, 64>(a, xre, xim, grid, stream);
+      case 3 * 2: return launch<3, 64>(a, xre, xim, grid, stream);
+      case 4 * 2: return launch<4, 64>(a, xre, xim, grid, stream);
+      case 1 * 2 + 1: return launch<1, 32>(a, xre, xim, grid, stream);
+      case 2 * 2 + 1: return launch<2, 32>(a, xre, xim, grid, stream);
+      case 3 * 2 + 1: return launch<3, 32>(a, xre, xim, grid, stream);
+      case 4 * 2 + 1: return launch<4, 32>(a, xre, xim, grid, stream);
+    }
+    return FAIRY2I_ERR_INVALID_ARG;
+  };
+  {
+    const int64_t tiles = (int64_t)count * ((n + 15) / 16) * ((B + tok - 1) / tok);
+    if (tiles > (int64_t(1) << 30)) return FAIRY2I_OK;
   }
   *handled = true;
-  switch (T * 2 + (tok == 32 ? 1 : 0)) {
-    case 1 * 2: return launch<1, 64>(a, xre, xim, grid, stream);
-    case 2 * 2: return launch<2, 64>(a, xre, xim, grid, stream);
-    case 3 * 2: return launch<3, 64>(a, xre, xim, grid, stream);
-    case 4 * 2: return launch<4, 64>(a, xre, xim, grid, stream);
-    case 1 * 2 + 1: return launch<1, 32>(a, xre, xim, grid, stream);
-    case 2 * 2 + 1: return launch<2, 32>(a, xre, xim, grid, stream);
-    case 3 * 2 + 1: return launch<3, 32>(a, xre, xim, grid, stream);
-    case 4 * 2 + 1: return launch<4, 32>(a, xre, xim, grid, stream);
+  // T = 3 at 16 rows per stage-matrix fills 96 of the 128 accumulator lanes; from
+  // kTwoLaunchMinTokens tokens on (where the MMAs, not the per-launch phases, set the time) it
+  // runs as stages 0-1 (32 rows each, every lane) and then stage 2 (64 rows) added into y.
+  if (T == 3 && B >= kTwoLaunchMinTokens) {
+    const fairy2i_status st = run(2, 0, 0);
+    if (st != FAIRY2I_OK) return st;
+    return run(1, 2, 1);
   }
-  *handled = false;
-  return FAIRY2I_OK;
+  return run(T, 0, 0);
 }
 
 fairy2i_status launch_wl_prefill(const void* x, fairy2i_dtype xdt, int64_t B, int64_t in_features,

@@ -327,6 +327,8 @@ def test_retired_path_2_is_rejected(F):
     # K split over CTA pairs (few tiles): 21 + 22 chunks, 2 + 3, 1 + 1, several tiles per pair
     (4096, 11008, 2, 64), (100, 1280, 4, 40), (130, 400, 1, 129), (11008, 4096, 3, 20),
     (1000, 2048, 1, 20), (4096, 4096, 1, 64), (200, 3008, 2, 7),
+    # T = 3 from 512 tokens on: a T = 2 launch, then a T = 1 launch adding into y
+    (300, 1024, 3, 600), (130, 400, 3, 512),
 ])
 def test_wl_tcgen05_prefill_path(F, out_f, in_f, T, B):
     """The tcgen05 prefill GEMM (path 3): ragged row blocks (R = 64, 32, 16, 16 rows of every
@@ -460,6 +462,7 @@ def test_group_prefill_path_any_batch(F, out_f, in_f, T, B, count):
     (4096, 4096, 2, 64, 3, torch.bfloat16),   # the 7B q/k/v at 64 tokens: 192 tiles, one launch
     (11008, 4096, 2, 64, 2, torch.bfloat16),  # gate / up at 64 tokens: K split, 4-5 tiles a pair
     (300, 512, 3, 130, 2, torch.bfloat16),    # ragged rows, three token tiles
+    (256, 512, 3, 520, 2, torch.bfloat16),    # T = 3 in two launches (stages 0-1, then 2)
     (37, 53, 2, 1, 4, torch.float32),         # fp32 x: members on the general path
 ])
 def test_wl_matmul_group_equals_separate_calls(F, out_f, in_f, T, B, count, dtype):
