@@ -68,8 +68,10 @@ constexpr int kGroupsPerCStage = 2 * kCChunks;
 constexpr int kRed = 4 * 16 * 2 * 128;            // floats: [sub-block][16 tokens][2][128 lanes]
 constexpr uint64_t kWaitNs = 1000000000ull;
 
-// Token-tile forms. TOK = 64: N = 128, one issuing thread per sign plane (the tensor pipe is the
-// bound). TOK = 32 (batches of at most 32 tokens): N = 64, two issuing threads per plane taking
+// Token-tile forms. TOK = 64: N = 128, one issuing thread per sign plane (each blocks ~200 cycles
+// on an MMA that keeps the tensor pipe ~64 cycles busy: the issue rate bounds the MMA phase; the
+// accumulators of more issuing threads would not leave tensor memory for the A ring).
+// TOK = 32 (batches of at most 32 tokens): N = 64, two issuing threads per plane taking
 // alternate groups, each into its own accumulator (an issuing thread blocks for about 150 cycles
 // on every MMA, so at the smaller N the issue rate is the bound); the epilogue adds the two in a
 // fixed order, so the result is deterministic.
