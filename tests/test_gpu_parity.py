@@ -434,6 +434,7 @@ def test_bounded_wait_latches_timeout_and_context_survives(F):
     (11008, 4096, 2, 8, 2),     # gate/up at 8 tokens
     (300, 1024, 3, 3, 2),       # ragged rows, T = 3
     (64, 256, 1, 2, 4),         # one 128-code chunk (no K split), four members
+    (256, 1024, 2, 16, 4),      # four members, 16 tiles: K split over CTA pairs
 ])
 def test_group_prefill_path_any_batch(F, out_f, in_f, T, B, count):
     """Path 3 for a group: one prefill GEMM launch holding every member's tiles, at skinny batches
