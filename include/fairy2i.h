@@ -174,9 +174,10 @@ fairy2i_status fairy2i_wl_matmul(const void* x, fairy2i_dtype xdt, int64_t B,
  *       the general kernel;
  *   2 = retired (an earlier tcgen05 decode kernel); returns FAIRY2I_ERR_INVALID_ARG;
  *   3 = the tcgen05 prefill GEMM (codes expanded into bf16 +-1 tiles in tensor memory, x by TMA,
- *       64 tokens per tile); it takes bf16 x with 16-byte aligned rows, ldx % 8 == 0,
- *       m % 8 == 0 (m = ceil(in_features/2)) and T <= 4, and returns FAIRY2I_ERR_INVALID_ARG for
- *       anything else;
+ *       64 tokens per tile, 32 up to B = 32; launches of few tiles split K over pairs of CTAs;
+ *       T = 3 from B = 512 on as a T = 2 and a T = 1 launch, the second adding into y); it takes
+ *       bf16 x with 16-byte aligned rows, ldx % 8 == 0, m % 8 == 0 (m = ceil(in_features/2)) and
+ *       T <= 4, and returns FAIRY2I_ERR_INVALID_ARG for anything else;
  *   4 = the persistent tcgen05 decode kernel (one CTA per SM looping over row blocks, the codes
  *       streamed through shared memory and decoded into tensor memory, K split over thread-block
  *       clusters of up to 8 CTAs whose partial rows are summed in rank order; one token: e2m1
@@ -193,7 +194,9 @@ fairy2i_status fairy2i_wl_matmul(const void* x, fairy2i_dtype xdt, int64_t B,
  * dependent launch): the codes must not be written by the kernel launched right before the
  * matmul on the same stream unless that kernel is one of this library's convert/quantize/adjoint
  * kernels, which end before any dependent kernel starts.
- * Results agree within the float32-accumulation tolerance whichever path runs. */
+ * Results agree within the float32-accumulation tolerance whichever path runs; every kernel sums
+ * in a fixed order, so a call repeated with the same shapes on the same device gives the same
+ * bits. */
 fairy2i_status fairy2i_wl_matmul_path(const void* x, fairy2i_dtype xdt, int64_t B,
                                       int64_t in_features, int64_t ldx, const uint32_t* codes,
                                       const float* scales, int64_t out_features, int T,
