@@ -74,9 +74,9 @@ DECODE_DRAM_BYTES = {
             "q": 4.231e6, "k": 4.231e6, "v": 4.231e6, "gate": 11.309e6, "up": 11.309e6},
     "stream": {"q,k,v": 12.655e6, "o": 4.265e6, "gate,up": 22.618e6, "down": 11.357e6},
 }
-PREFILL_T2_UP_DRAM_BYTES = 28.110e6 + 37.261e6
+PREFILL_T2_UP_DRAM_BYTES = 28.121e6 + 36.813e6
 # ncu sm__pipe_tensor_cycles_active of the same prefill launch (T = 2, up layer, 2048 tokens)
-PREFILL_T2_UP_TENSOR_PIPE_PCT = 54.5
+PREFILL_T2_UP_TENSOR_PIPE_PCT = 54.9
 
 
 def decode_kernel(c, path, sms):
