@@ -258,6 +258,18 @@ def make_calls(linears, B: int, dev, groups=GROUPS):
     return calls, x_all, y_all
 
 
+def step_launches(ncalls: int, B: int, path: int, T: int = T_STAGES) -> int:
+    """Kernel launches of one step of `ncalls` (grouped) bf16 calls: one per call on the automatic
+    path (B = 1 on a decode kernel, 2 <= B <= 4 on the chained kernel, larger batches on the
+    prefill GEMM, T = 3 from 512 tokens on as two launches); one per call and per 4 tokens on the
+    chained kernel chosen explicitly (path 5)."""
+    if path == 5:
+        return ncalls * ((B + 3) // 4)
+    if T == 3 and B >= 512:
+        return 2 * ncalls
+    return ncalls
+
+
 def call_bytes(c, B):
     """Algorithmic bytes of one call: every member's codes, scales and y, the shared x once."""
     per = [layer_bytes(m["rows"], m["cols"], B) for m in c["members"]]
@@ -316,10 +328,7 @@ def run_ours(args, world, rank, local):
     calls, x_all, y_all = make_calls(linears, B, dev, groups)
     step_bytes = sum(call_bytes(c, B) for c in calls)
     nlinears = sum(len(c["members"]) for c in calls)
-    # a grouped call is one launch: B = 1 on a decode kernel, 2 <= B <= 4 on the chained kernel,
-    # larger batches on the prefill GEMM; on the chained kernel chosen explicitly (path 5) one
-    # launch per 4 tokens
-    launches_per_step = (len(calls) * ((B + 3) // 4) if args.decode_path == 5 else len(calls))
+    launches_per_step = step_launches(len(calls), B, args.decode_path)
 
     def step():
         for c in calls:

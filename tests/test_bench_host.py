@@ -66,3 +66,14 @@ def test_decode_bytes_per_step():
     assert total == 1_625_938_944
     codes = 32 * sum(2 * 2 * ((r + 1) // 2) * ((c + 1) // 2) // 4 for (_, r, c) in synth.PROJECTIONS)
     assert codes == 1_619_001_344   # T = 2 bits per real parameter of the 7B linears
+
+
+def test_step_launches_follow_the_automatic_path():
+    """One launch per grouped call on the automatic path at every batch the bench runs, the
+    chained kernel's explicit path one per 4 tokens, T = 3 from 512 tokens two per call."""
+    for B in (1, 2, 4, 5, 8, 16, 64, 2048):
+        assert bench.step_launches(128, B, 0) == 128
+    assert bench.step_launches(128, 8, 5) == 256
+    assert bench.step_launches(128, 3, 5) == 128
+    assert bench.step_launches(4, 512, 0, T=3) == 8
+    assert bench.step_launches(4, 511, 0, T=3) == 4
